@@ -1,0 +1,207 @@
+/*
+ * sva.h -- streaming video attention: policy-indexed chunk-causal attention
+ * over a (chunk, level)-indexed KV cache, with a fused 3D-RoPE + cache
+ * scatter, for one GB300 GPU (sm_103a).
+ *
+ * Method: "Rethinking Streaming Video Diffusion Model: Context, Execution,
+ * and Training", Section 3.  A *node* (b, j) is chunk b of the video at
+ * denoising level j in {0..K} (j = K pure noise, j = 0 clean; Section 3.1).
+ * A context policy phi picks, for every history offset r in
+ * {1..min(W, b-1)}, the level of chunk b-r the node reads (Eq. 2-3); the
+ * node's queries then attend over its own chunk (bidirectionally) plus the
+ * cached keys/values of those states, everything else masked with -inf
+ * (Eq. 4).  Several nodes of one pipeline round (Eq. 6) are processed by one
+ * launch, which is how progressive history is executed (Section 3.3).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Every device buffer is owned by the caller: the cache buffer handed to
+ *   sva_cache_create and every Q/K/V/O/LSE tensor.  The library owns only
+ *   the opaque sva_cache object (host slot table and cached TMA
+ *   descriptors), freed by sva_destroy.  The library never allocates device
+ *   memory.
+ * - Tensors are dense, row-major, bf16 unless stated, 16-byte aligned.
+ *   Token-major activations are [n_nodes][T][H][d] with T = F*Hp*Wp tokens
+ *   per chunk, token u = (f*Hp + h)*Wp + w.
+ * - Calls that take a stream validate on the host, enqueue on that stream and
+ *   return; nothing is launched when validation fails.  Device-side errors
+ *   (a bounded wait inside a kernel that timed out) are reported later by
+ *   sva_poll_device_status.
+ * - On failure a call returns a non-zero sva_status and sets a thread-local
+ *   message readable with sva_last_error().
+ * - One cache is used from one host thread and one stream at a time.
+ */
+#ifndef SVA_H_
+#define SVA_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  SVA_OK = 0,
+  SVA_ERR_INVALID_ARGUMENT = 1, /* null/misaligned pointer, bad size, bad id */
+  SVA_ERR_NOT_RESIDENT = 2,     /* a (seq, chunk, level) state is not in the cache */
+  SVA_ERR_CAUSALITY = 3,        /* a context state is not in the node's past (Eq. 4) */
+  SVA_ERR_CAPACITY = 4,         /* too many nodes/contexts/slots, position beyond the table */
+  SVA_ERR_UNSUPPORTED = 5,      /* geometry the kernels do not implement */
+  SVA_ERR_CUDA = 6,             /* a CUDA runtime/driver call failed */
+  SVA_ERR_DEVICE_TIMEOUT = 7,   /* a kernel's bounded wait expired */
+  SVA_ERR_UNAVAILABLE = 8       /* a selected level not yet reached by the pipeline (Eq. 7) */
+} sva_status;
+
+/* Context policies, Eq. 3 (Section 3.2). */
+enum {
+  SVA_POLICY_CLEAN = 0, /* phi(j, r) = 0 */
+  SVA_POLICY_SAME = 1,  /* phi(j, r) = j */
+  SVA_POLICY_PROG = 2   /* phi(j, r) = max(j - r, 0) */
+};
+
+#define SVA_MAX_CTX 16   /* history states one node may read */
+#define SVA_MAX_NODES 64 /* nodes in one sva_rope_kv_write / sva_attend_nodes call */
+
+typedef struct sva_cache sva_cache;
+typedef struct CUstream_st* sva_stream; /* a cudaStream_t; NULL = legacy default stream */
+
+/* Geometry of the chunks and of the KV cache.
+ *   num_heads   H, 1..128
+ *   head_dim    d, 64 or 128
+ *   frames      F latent frames per chunk; grid_h x grid_w patches per frame
+ *               (T = F*grid_h*grid_w tokens per chunk, 1..65536)
+ *   num_slots   number of (chunk, level) states the cache holds at once
+ *   rope_pairs  head-dimension pairs rotated by the t, h and w positions;
+ *               they must sum to d/2 (3D RoPE reading: the paper does not name
+ *               a positional encoding)
+ *   max_frames  absolute latent-frame positions covered by the RoPE table:
+ *               every written chunk b needs F*b + F - 1 < max_frames
+ *   rope_theta  RoPE base (10000 in the usual convention)              */
+typedef struct {
+  int32_t num_heads;
+  int32_t head_dim;
+  int32_t frames;
+  int32_t grid_h;
+  int32_t grid_w;
+  int32_t num_slots;
+  int32_t rope_pairs[3];
+  int32_t max_frames;
+  double rope_theta;
+} sva_geometry;
+
+/* One denoising node of a launch (Section 3.1-3.3).
+ *   seq          independent video stream the node belongs to (stream
+ *                batching); contexts must come from the same seq
+ *   chunk, level the node (b, j)
+ *   own_slot     cache slot bound to (seq, chunk, level); written by
+ *                sva_rope_kv_write, always visible to the node itself
+ *   n_ctx        number of history states read, 0..SVA_MAX_CTX
+ *   ctx_slot     their cache slots (e.g. from sva_select_context +
+ *                sva_cache_lookup), each of a chunk < `chunk`
+ *   ctx_visible  Eq. 4 at state granularity: 1 = mask 0 on that state's
+ *                tokens, 0 = mask -inf (the state is skipped)           */
+typedef struct {
+  int32_t seq;
+  int32_t chunk;
+  int32_t level;
+  int32_t own_slot;
+  int32_t n_ctx;
+  int32_t ctx_slot[SVA_MAX_CTX];
+  uint8_t ctx_visible[SVA_MAX_CTX];
+} sva_node;
+
+/* Bytes of device memory the cache needs for `g`: the slot pool
+ * [num_slots][2 (K, V)][H][Tpad][d] bf16 with Tpad = T rounded up to 128,
+ * the RoPE cos/sin tables and a status word.  0 if `g` is invalid. */
+size_t sva_cache_bytes(const sva_geometry* g);
+
+/* Creates a cache over the caller's device buffer `dev_buf` (at least
+ * sva_cache_bytes(g) bytes, 256-byte aligned, on the current device).
+ * Zeroes the pad rows and the status word, uploads the RoPE tables, and
+ * builds the TMA descriptor of the slot pool.  Synchronous.  The buffer must
+ * outlive the cache.  Errors: INVALID_ARGUMENT, UNSUPPORTED, CUDA. */
+sva_status sva_cache_create(const sva_geometry* g, void* dev_buf, size_t bytes, sva_cache** out);
+
+/* Binds a free slot to state (seq, chunk, level) (the KV cache of
+ * Section 3.2, indexed by chunk and level).  The slot is not resident until
+ * sva_rope_kv_write has written it.  Errors: INVALID_ARGUMENT (level < 0 or
+ * the state is already bound), CAPACITY (no free slot). */
+sva_status sva_cache_bind(sva_cache* c, int32_t seq, int32_t chunk, int32_t level, int32_t* slot);
+
+/* Slot bound to (seq, chunk, level).  Errors: NOT_RESIDENT if unbound. */
+sva_status sva_cache_lookup(const sva_cache* c, int32_t seq, int32_t chunk, int32_t level,
+                            int32_t* slot);
+
+/* Frees the slot of (seq, chunk, level) (rolling window).  Host-side only:
+ * the caller must not release a slot that a queued kernel still reads.
+ * Errors: NOT_RESIDENT if unbound. */
+sva_status sva_cache_release(sva_cache* c, int32_t seq, int32_t chunk, int32_t level);
+
+/* Eq. 2-3 (Section 3.2) with the full offset window R = {1..min(W, b-1)}:
+ * writes (chunk - r, phi(level, r)) for r = 1.. into chunks/levels, in order
+ * of increasing r, and their number into *n.  Chunks are numbered from 1 as
+ * in the paper.  Errors: INVALID_ARGUMENT (unknown policy, K < 1,
+ * level outside 0..K, W < 0, null pointers), CAPACITY (cap too small). */
+sva_status sva_select_context(int32_t policy, int32_t K, int32_t W, int32_t chunk, int32_t level,
+                              int32_t cap, int32_t* chunks, int32_t* levels, int32_t* n);
+
+/* Eq. 6 (Section 3.3): the states [x_n^K, x_{n-1}^{K-1}, ..., x_{n-K+1}^1]
+ * active at the start of round n of a pipeline over chunks 1..B, chunks
+ * outside 1..B left out.  Writes them (levels K down to 1) and their number.
+ * Errors: INVALID_ARGUMENT, CAPACITY (cap < number of states). */
+sva_status sva_pipeline_round(int32_t K, int32_t B, int32_t round, int32_t cap, int32_t* chunks,
+                              int32_t* levels, int32_t* count);
+
+/* Eq. 7 (Section 3.3): checks that every state (chunks[i], levels[i]) a node
+ * (chunk, level) of a K-level pipeline reads has been reached, i.e.
+ * levels[i] >= max(level - r, 0) with r = chunk - chunks[i] >= 1.
+ * Returns OK, UNAVAILABLE (first violation named in sva_last_error), or
+ * INVALID_ARGUMENT / CAUSALITY for malformed lists. */
+sva_status sva_check_pipeline(int32_t K, int32_t level, int32_t chunk, int32_t n,
+                              const int32_t* chunks, const int32_t* levels);
+
+/* Applies 3D RoPE to each node's new keys (and, if q_inout is not NULL, to
+ * its queries, in place) at the node's absolute positions (F*chunk + f, h, w)
+ * and scatters K' and the unrotated V into the node's own slot (the cache
+ * write that makes the node's features available to later reads and to
+ * in-round progressive reads, Section 3.3).  Marks the own slots resident.
+ *   k_new, v_new, q_inout: [n_nodes][T][H][d] bf16, node i = nodes[i].
+ * Stream-ordered.  Errors: INVALID_ARGUMENT (null/misaligned pointer,
+ * unbound or mismatched own_slot, duplicate own_slot), CAPACITY
+ * (n_nodes > SVA_MAX_NODES, position beyond max_frames), CUDA. */
+sva_status sva_rope_kv_write(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
+                             const void* k_new, const void* v_new, void* q_inout, sva_stream s);
+
+/* Policy-indexed chunk-causal attention (Eq. 4) for a batch of nodes:
+ *   out[i][u][h] = sum_v softmax_v(scale * q[i][u][h] . k_v + M(u, v)) v_v
+ * over the keys of node i's own slot and its visible context slots; M is 0
+ * on those and -inf elsewhere; attention inside the own chunk is
+ * bidirectional.
+ *   q    [n_nodes][T][H][d] bf16 (already rotated)
+ *   out  [n_nodes][T][H][d] bf16
+ *   lse  [n_nodes][H][T] fp32 natural-log sum-exp of the masked logits, or NULL
+ *   scale  logit scale, e.g. 1/sqrt(d); finite and > 0
+ * Every referenced slot must be resident; contexts must be of the same seq
+ * and an earlier chunk, with no slot repeated.  Stream-ordered after the
+ * sva_rope_kv_write that filled the slots.  Errors: INVALID_ARGUMENT,
+ * NOT_RESIDENT, CAUSALITY, CAPACITY, CUDA. */
+sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* q,
+                            void* out, float* lse, float scale, sva_stream s);
+
+/* Synchronizes `s`, then reads and clears the device status word: returns
+ * DEVICE_TIMEOUT if a kernel gave up a bounded wait since the last poll,
+ * CUDA if the stream reported an error, else OK. */
+sva_status sva_poll_device_status(sva_cache* c, sva_stream s);
+
+/* Frees the cache object (not the caller's device buffer). */
+sva_status sva_destroy(sva_cache* c);
+
+/* Thread-local message describing the last failure ("" if none). */
+const char* sva_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SVA_H_ */

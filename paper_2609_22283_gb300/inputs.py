@@ -1,0 +1,164 @@
+"""Workload descriptions and seeded synthetic inputs.
+
+This module is the only code the CUDA path and the CPU oracle share.  It
+holds data and random numbers, none of the method's arithmetic: no context
+selection, no RoPE, no attention.  Each workload lists its nodes and the
+states already in the cache as plain data (derived by hand from the
+progressive, same-level and clean rules of Eq. 3 and written out here); the
+library and the oracle each derive the context lists themselves.
+
+Synthetic inputs stand in for the paper's video latents (Wan2.1 geometry,
+832x480 at 16 FPS, 3-latent-frame chunks, Section 4 and Appendix A): every
+tensor is drawn from a seeded torch CPU generator as N(0, 1) fp32 and rounded
+to bf16, in this order: for each prefilled state (in the listed order) its K
+then its V [T][H][d]; then Q, K_new and V_new [n_nodes][T][H][d].  With
+`outliers`, each draw is followed by a U(0, 1) draw of the same shape on the
+same generator and elements whose uniform is below 0.01 are multiplied by 10.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+
+import torch
+
+
+def rope_pairs_for(d: int) -> tuple[int, int, int]:
+    """Head-dimension pairs given to the t, h and w axes: h and w get
+    floor(d/6) pairs each, t the rest (22/21/21 for d = 128, 12/10/10 for 64)."""
+    hw = d // 6
+    return (d // 2 - 2 * hw, hw, hw)
+
+
+@dataclass(frozen=True)
+class Workload:
+    name: str
+    seed: int
+    F: int            # latent frames per chunk
+    Hp: int           # patch rows per frame
+    Wp: int           # patch columns per frame
+    H: int            # attention heads
+    d: int            # head dim
+    K: int            # denoising levels (node levels 1..K, clean level 0)
+    W: int            # history window in chunks
+    policy: str       # "clean" | "same" | "prog"
+    nodes: tuple      # ((seq, chunk, level), ...) processed by the step
+    prefilled: tuple  # ((seq, chunk, level), ...) states cached before the step
+    outliers: bool = False
+    B: int = 40       # chunks in the video (pipeline length, Eq. 6)
+    round: int | None = None  # pipeline round the nodes form (Eq. 6), if any
+    description: str = ""
+    theta: float = 10000.0
+    pairs: tuple = field(default=None)
+
+    def __post_init__(self):
+        if self.pairs is None:
+            object.__setattr__(self, "pairs", rope_pairs_for(self.d))
+
+    @property
+    def T(self) -> int:
+        return self.F * self.Hp * self.Wp
+
+    @property
+    def n_nodes(self) -> int:
+        return len(self.nodes)
+
+    @property
+    def states(self) -> tuple:
+        """Every state the step touches: prefilled ones, then the nodes' own."""
+        return tuple(self.prefilled) + tuple(self.nodes)
+
+    @property
+    def max_frames(self) -> int:
+        last = max(c for (_, c, _) in self.states)
+        return self.F * (last + 1) + self.F
+
+
+def _round_nodes(seq: int, K: int, n: int):
+    # written out by hand: chunk n - K + j at level j, for j = K .. 1 (Eq. 6)
+    return tuple((seq, n - K + j, j) for j in range(K, 0, -1))
+
+
+_PROG_PREFILL_20 = tuple((0, c, 0) for c in range(11, 17))      # chunks 11..16, clean
+_SAME_PREFILL_20 = tuple((0, b - r, j) for (_, b, j) in _round_nodes(0, 4, 20) for r in (1, 2, 3))
+
+WORKLOADS = {
+    "tiny": Workload(
+        name="tiny", seed=0, F=1, Hp=8, Wp=8, H=2, d=64, K=2, W=2, policy="prog",
+        nodes=((0, 3, 2), (0, 2, 1)), prefilled=((0, 1, 0),), B=3, round=3,
+        description="3 chunks x 64 tokens (1 latent frame of 8x8), K=2, 2 nodes (3,2),(2,1) "
+                    "batched, 2 heads x 64, progressive history, W=2"),
+    "clean1": Workload(
+        name="clean1", seed=1, F=3, Hp=30, Wp=52, H=12, d=128, K=4, W=3, policy="clean",
+        nodes=((0, 20, 4),), prefilled=((0, 17, 0), (0, 18, 0), (0, 19, 0)),
+        description="1 node (20,4), clean history W=3: 4680 queries x 12 heads x 128 over "
+                    "4680 own + 3x4680 clean history keys (Lkv 18720)"),
+    "same4": Workload(
+        name="same4", seed=2, F=3, Hp=30, Wp=52, H=12, d=128, K=4, W=3, policy="same",
+        nodes=_round_nodes(0, 4, 20), prefilled=_SAME_PREFILL_20, round=20,
+        description="round 20 of a K=4 pipeline: nodes (20,4),(19,3),(18,2),(17,1), same-level "
+                    "history W=3 (Lkv 18720), 12 heads x 128"),
+    "prog4": Workload(
+        name="prog4", seed=3, F=3, Hp=30, Wp=52, H=12, d=128, K=4, W=6, policy="prog",
+        nodes=_round_nodes(0, 4, 20), prefilled=_PROG_PREFILL_20, round=20,
+        description="round 20 of a K=4 pipeline: nodes (20,4),(19,3),(18,2),(17,1), progressive "
+                    "history W=6 (7-chunk window, Lkv 32760), in-round reads, 12 heads x 128"),
+    "stress14b": Workload(
+        name="stress14b", seed=4, F=3, Hp=30, Wp=52, H=40, d=128, K=4, W=6, policy="prog",
+        nodes=_round_nodes(0, 4, 20) + _round_nodes(1, 4, 20),
+        prefilled=_PROG_PREFILL_20 + tuple((1, c, l) for (_, c, l) in _PROG_PREFILL_20),
+        outliers=True, round=20,
+        description="2 video streams x the prog4 round: 8 nodes, 40 heads x 128, Lkv 32760, "
+                    "N(0,1) with 1% x10 outliers"),
+}
+
+# The order the workloads are listed in the task's configuration table.
+ORDER = ("tiny", "clean1", "same4", "prog4", "stress14b")
+
+
+@dataclass
+class Inputs:
+    history: dict      # {(seq, chunk, level): (K_raw, V_raw)} bf16 [T][H][d]
+    q: torch.Tensor    # bf16 [n][T][H][d]
+    k_new: torch.Tensor
+    v_new: torch.Tensor
+
+
+def generate(w: Workload) -> Inputs:
+    g = torch.Generator(device="cpu")
+    g.manual_seed(w.seed)
+
+    def draw(shape):
+        x = torch.randn(shape, generator=g, dtype=torch.float32)
+        if w.outliers:
+            u = torch.rand(shape, generator=g, dtype=torch.float32)
+            x = torch.where(u < 0.01, x * 10.0, x)
+        return x.to(torch.bfloat16)
+
+    T, H, d, n = w.T, w.H, w.d, w.n_nodes
+    history = {}
+    for s in w.prefilled:
+        k = draw((T, H, d))
+        v = draw((T, H, d))
+        history[tuple(s)] = (k, v)
+    q = draw((n, T, H, d))
+    k_new = draw((n, T, H, d))
+    v_new = draw((n, T, H, d))
+    return Inputs(history, q, k_new, v_new)
+
+
+def all_states(w: Workload, inp: Inputs) -> dict:
+    """{(seq, chunk, level): (K_raw, V_raw)} for prefilled states and nodes' own states."""
+    st = dict(inp.history)
+    for i, s in enumerate(w.nodes):
+        st[tuple(s)] = (inp.k_new[i], inp.v_new[i])
+    return st
+
+
+def sample_rows(w: Workload, count: int, seed: int = 1234):
+    """Seeded query rows for sampled parity, always including the tile edges."""
+    T = w.T
+    edges = sorted({0, 1, 63, 64, 127, 128, T - 73, T - 72, T - 1} & set(range(T)))
+    g = torch.Generator(device="cpu")
+    g.manual_seed(seed)
+    extra = torch.randperm(T, generator=g)[:count].tolist()
+    return sorted(set(edges) | set(extra))

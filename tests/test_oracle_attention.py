@@ -1,0 +1,164 @@
+"""Pins of the oracle's masked softmax attention (Eq. 4) and of its per-node
+pipeline (selection + RoPE + bf16 store + attention): against the dense-mask
+brute force over the whole (chunk, level) grid, softmax invariants, library
+routines (scipy softmax / logsumexp, torch SDPA in fp64) and row
+independence."""
+import math
+
+import numpy as np
+import pytest
+import scipy.special
+import torch
+
+from paper_2609_22283_gb300 import inputs as I
+
+
+def _tiny(oracle_mod):
+    w = I.WORKLOADS["tiny"]
+    inp = I.generate(w)
+    g = oracle_mod.Geometry(F=w.F, Hp=w.Hp, Wp=w.Wp, H=w.H, d=w.d, pairs=w.pairs, theta=w.theta)
+    return w, inp, g
+
+
+def _f64(t):
+    return t.to(torch.float64).numpy()
+
+
+def test_tiny_against_dense_brute_force(oracle_mod):
+    from oracle import brute
+    w, inp, g = _tiny(oracle_mod)
+    states = {k: (_f64(a), _f64(b)) for k, (a, b) in I.all_states(w, inp).items()}
+    # distractors the policy must NOT select: other levels of past chunks, a
+    # future chunk, and the same chunks of another sequence
+    rng = np.random.default_rng(7)
+    grid = dict(states)
+    for s in [(0, 1, 1), (0, 1, 2), (0, 2, 0), (0, 2, 2), (0, 4, 0), (1, 1, 0), (1, 2, 1)]:
+        grid[s] = (rng.standard_normal((w.T, w.H, w.d)), rng.standard_normal((w.T, w.H, w.d)))
+    scale = 1.0 / math.sqrt(w.d)
+    for i, node in enumerate(w.nodes):
+        q = _f64(inp.q[i])
+        out, lse, _ = oracle_mod.node_forward(g, oracle_mod.POLICY_IDS[w.policy], w.W, node,
+                                              states, q, range(w.H), range(w.T), scale)
+        bo, bl = brute.brute_forward(w.policy, w.W, w.F, w.Hp, w.Wp, w.pairs, w.theta, node,
+                                     grid, q, range(w.H), scale)
+        np.testing.assert_allclose(out, bo, rtol=0, atol=1e-12)
+        np.testing.assert_allclose(lse, bl, rtol=0, atol=1e-12)
+
+
+def test_hidden_state_matches_brute_force(oracle_mod):
+    from oracle import brute
+    w, inp, g = _tiny(oracle_mod)
+    states = {k: (_f64(a), _f64(b)) for k, (a, b) in I.all_states(w, inp).items()}
+    node = w.nodes[0]                      # (3, 2) reads (2, 1) and (1, 0)
+    hidden = frozenset({(2, 1)})
+    q = _f64(inp.q[0])
+    scale = 0.2
+    out, lse, _ = oracle_mod.node_forward(g, oracle_mod.POLICY_IDS[w.policy], w.W, node, states, q,
+                                          [1], range(w.T), scale, hidden=hidden)
+    bo, bl = brute.brute_forward(w.policy, w.W, w.F, w.Hp, w.Wp, w.pairs, w.theta, node, states, q,
+                                 [1], scale, hidden=hidden)
+    np.testing.assert_allclose(out, bo, rtol=0, atol=1e-12)
+    full, _, _ = oracle_mod.node_forward(g, oracle_mod.POLICY_IDS[w.policy], w.W, node, states, q,
+                                         [1], range(w.T), scale)
+    assert not np.allclose(out, full)
+
+
+def test_rows_are_the_library_softmax(oracle_mod):
+    rng = np.random.default_rng(0)
+    L, d = 48, 64
+    q = rng.standard_normal((10, d))
+    k = rng.standard_normal((L, d))
+    v = np.eye(L, d)                        # one-hot values: out = attention weights
+    mask = np.where(rng.random(L) < 0.3, -np.inf, 0.0)
+    scale = 0.37
+    out, lse = oracle_mod.attend_rows(q, k, v, scale, mask)
+    logits = scale * q @ k.T + mask
+    ref = scipy.special.softmax(logits, axis=1)
+    np.testing.assert_allclose(out[:, :L], ref, rtol=1e-13, atol=1e-15)
+    np.testing.assert_allclose(out.sum(axis=1), 1.0, rtol=1e-13)
+    assert np.all(out[:, :L][:, mask == -np.inf] == 0.0)
+    np.testing.assert_allclose(lse, scipy.special.logsumexp(logits, axis=1), rtol=1e-13)
+
+
+def test_constant_values_and_identical_keys(oracle_mod):
+    rng = np.random.default_rng(1)
+    L, d = 300, 128
+    q = rng.standard_normal((7, d)) * 3
+    k = rng.standard_normal((L, d))
+    v = np.full((L, d), 0.625)
+    out, _ = oracle_mod.attend_rows(q, k, v, 0.1)
+    np.testing.assert_allclose(out, 0.625, rtol=1e-14)
+    k_same = np.tile(rng.standard_normal(d), (L, 1))
+    v = rng.standard_normal((L, d))
+    mask = np.where(np.arange(L) % 3 == 0, -np.inf, 0.0)
+    out, lse = oracle_mod.attend_rows(q, k_same, v, 0.1, mask)
+    np.testing.assert_allclose(out, np.tile(v[mask == 0].mean(axis=0), (7, 1)), rtol=1e-12, atol=1e-14)
+
+
+def test_fully_masked_row_reading(oracle_mod):
+    q = np.ones((2, 64))
+    k = np.ones((5, 64))
+    v = np.ones((5, 64))
+    out, lse = oracle_mod.attend_rows(q, k, v, 1.0, np.full(5, -np.inf))
+    assert np.all(out == 0.0) and np.all(lse == -np.inf)
+
+
+def test_clean_single_node_is_block_causal_sdpa(oracle_mod):
+    """Clean policy, one node: the node's rows equal the last block of ordinary
+    block-causal attention over [x_{b-W}^0, ..., x_{b-1}^0, x_b^j] (fp64 torch SDPA)."""
+    F, Hp, Wp, H, d, W = 1, 4, 6, 2, 64, 3
+    pairs = I.rope_pairs_for(d)
+    g = oracle_mod.Geometry(F=F, Hp=Hp, Wp=Wp, H=H, d=d, pairs=pairs)
+    T = g.T
+    b, j = 9, 3
+    rng = np.random.default_rng(3)
+    bfr = lambda x: oracle_mod.bf16(x)
+    states = {}
+    for c in range(b - W, b):
+        states[(0, c, 0)] = (bfr(rng.standard_normal((T, H, d))), bfr(rng.standard_normal((T, H, d))))
+    states[(0, b, j)] = (bfr(rng.standard_normal((T, H, d))), bfr(rng.standard_normal((T, H, d))))
+    # states the clean policy must ignore
+    for c in range(b - W, b):
+        states[(0, c, j)] = (bfr(rng.standard_normal((T, H, d))), bfr(rng.standard_normal((T, H, d))))
+    q_raw = bfr(rng.standard_normal((T, H, d)))
+    scale = 1 / math.sqrt(d)
+    out, lse, sel = oracle_mod.node_forward(g, oracle_mod.POLICY_CLEAN, W, (0, b, j), states, q_raw,
+                                            range(H), range(T), scale)
+    assert sel == [(b - r, 0) for r in range(1, W + 1)]
+    order = [(c, 0) for c in range(b - W, b)] + [(b, j)]
+    for h in range(H):
+        ks = [oracle_mod.bf16(oracle_mod.rope_head(states[(0,) + s][0][:, h, :], s[0], g)) for s in order]
+        vs = [states[(0,) + s][1][:, h, :] for s in order]
+        qs = [oracle_mod.bf16(oracle_mod.rope_head(np.zeros((T, d)), s[0], g)) for s in order[:-1]]
+        qs.append(oracle_mod.bf16(oracle_mod.rope_head(q_raw[:, h, :], b, g)))
+        Q = torch.from_numpy(np.concatenate(qs))[None, None]
+        K = torch.from_numpy(np.concatenate(ks))[None, None]
+        V = torch.from_numpy(np.concatenate(vs))[None, None]
+        blk = torch.arange(len(order) * T) // T
+        allowed = blk[:, None] >= blk[None, :]                     # block-causal
+        ref = torch.nn.functional.scaled_dot_product_attention(Q, K, V, attn_mask=allowed, scale=scale)
+        np.testing.assert_allclose(out[h], ref[0, 0, -T:].numpy(), rtol=1e-12, atol=1e-13)
+
+
+def test_rows_independent(oracle_mod):
+    """Computing a subset of rows gives the same numbers as computing all rows."""
+    w, inp, g = _tiny(oracle_mod)
+    states = {k: (_f64(a), _f64(b)) for k, (a, b) in I.all_states(w, inp).items()}
+    q = _f64(inp.q[0])
+    scale = 0.125
+    full, fl, _ = oracle_mod.node_forward(g, 2, w.W, w.nodes[0], states, q, [0, 1], range(w.T), scale)
+    rows = [5, 0, 63, 17]
+    part, pl, _ = oracle_mod.node_forward(g, 2, w.W, w.nodes[0], states, q, [1], rows, scale)
+    np.testing.assert_array_equal(part[0], full[1][rows])
+    np.testing.assert_array_equal(pl[0], fl[1][rows])
+
+
+@pytest.mark.parametrize("name", ["clean1", "prog4"])
+def test_full_geometry_selection_is_prefilled(oracle_mod, name):
+    """Every state a workload's nodes select is either prefilled or written by
+    a node of the same step (the in-round progressive reads)."""
+    w = I.WORKLOADS[name]
+    have = set(w.states)
+    for (s, b, j) in w.nodes:
+        for (c, lvl) in oracle_mod.select(oracle_mod.POLICY_IDS[w.policy], w.W, b, j):
+            assert (s, c, lvl) in have
