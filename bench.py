@@ -1,0 +1,424 @@
+#!/usr/bin/env python3
+"""Benchmark of the hot path: policy-indexed chunk-causal attention with its
+fused 3D-RoPE + KV-cache write, on seeded synthetic inputs shaped like the
+paper's workloads (Wan2.1 geometry, 3-latent-frame chunks of 30x52 patches).
+
+One step = one pass of the whole path over one launch's nodes: context
+selection and availability check on the host, sva_rope_kv_write, and
+sva_attend_nodes, with inputs resident in HBM.  The L2 is flushed (256 MiB
+write) between timed steps, outside the timed intervals.  `value` is the
+attention's algorithmic TFLOP/s over whole steps (4*T*Lkv*d*H per node).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+  python bench.py --impl reference ...   # the fp64 CPU oracle on the same workload
+
+Under torchrun (N > 1) each rank runs an independent replica of the workload
+on its own GPU (the path has no exchange step); the step time is the max over
+ranks and `value` counts the work of all ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "chunk-attention TFLOP/s (% of GB300 BF16 peak) and denoising nodes/s per layer"
+DEFAULT_WORKLOAD = "clean1"
+KERNEL_SOURCES = ["paper_2609_22283_gb300/csrc/attend.cu", "paper_2609_22283_gb300/csrc/ptx.cuh",
+                  "paper_2609_22283_gb300/csrc/internal.h"]
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "attend_dram_traffic.md")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def attn_flops(w) -> float:
+    """Algorithmic FLOPs of one step's attention: 4*T*Lkv*d*H per node (QK^T + PV)."""
+    total = 0.0
+    for (_, b, _) in w.nodes:
+        n_ctx = max(0, min(w.W, b - 1))
+        total += 4.0 * w.T * (1 + n_ctx) * w.T * w.d * w.H
+    return total
+
+
+def rope_bytes(w) -> float:
+    """Algorithmic bytes of one rope_kv_write launch: K, V, Q read once, written once."""
+    return 3 * 2 * w.n_nodes * w.T * w.H * w.d * 2.0
+
+
+def kernel_hash() -> str:
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        with open(os.path.join(ROOT, f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def read_traffic(workload: str):
+    """DRAM bytes per attend launch from the committed ncu summary, if it was
+    taken on the current kernel source (matching hash); else None."""
+    try:
+        text = open(TRAFFIC_FILE).read()
+    except OSError:
+        return None
+    want = kernel_hash()
+    for line in text.splitlines():
+        parts = [p.strip() for p in line.strip().strip("|").split("|")]
+        if len(parts) >= 3 and parts[0] == workload and parts[1] == want:
+            try:
+                return float(parts[2])
+            except ValueError:
+                return None
+    return None
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return p, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.QUERY}", "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", str(self.index)],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, f[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return None
+        sm.sort()
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        import torch
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+    return world, rank, local
+
+
+def reduce_max(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    dev = torch.device("cuda") if torch.cuda.is_available() and dist.get_backend() == "nccl" else torch.device("cpu")
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ---------------------------------------------------------------- oracle (CPU)
+
+def oracle_sample(w, inp, seconds: float, min_rows: int = 16):
+    """Times the fp64 oracle on node 0, head 0, growing batches of seeded query
+    rows until about `seconds` of CPU work; returns (TFLOP/s, rows, secs, cores)."""
+    import numpy as np
+    import torch
+    import oracle
+    from paper_2609_22283_gb300 import inputs as I
+
+    oracle.build()
+    g = oracle.Geometry(F=w.F, Hp=w.Hp, Wp=w.Wp, H=w.H, d=w.d, pairs=w.pairs, theta=w.theta)
+    states = {k: (a.to(torch.float64).numpy(), b.to(torch.float64).numpy())
+              for k, (a, b) in I.all_states(w, inp).items()}
+    (_, b, _) = w.nodes[0]
+    lkv = w.T * (1 + max(0, min(w.W, b - 1)))
+    q = inp.q[0].to(torch.float64).numpy()
+    rng = np.random.default_rng(5)
+    rows_done, spent = 0, 0.0
+    batch = min_rows
+    while spent < seconds:
+        rows = sorted(rng.choice(w.T, size=min(batch, w.T), replace=False).tolist())
+        t0 = time.perf_counter()
+        oracle.node_forward(g, oracle.POLICY_IDS[w.policy], w.W, w.nodes[0], states, q, [0], rows,
+                            1.0 / math.sqrt(w.d))
+        spent += time.perf_counter() - t0
+        rows_done += len(rows)
+        batch = min(w.T, batch * 2)
+    flops = 4.0 * rows_done * lkv * w.d
+    return flops / spent / 1e12, rows_done, spent, oracle.num_threads()
+
+
+def run_reference(args, world, rank):
+    """The reference arm: the fp64 CPU oracle, as it stands, on the same workload."""
+    if rank != 0:
+        return 0
+    from paper_2609_22283_gb300 import inputs as I
+    w = I.WORKLOADS[args.workload]
+    inp = I.generate(w)
+    per_step = args.reference_seconds
+    for _ in range(args.warmup):
+        oracle_sample(w, inp, per_step / 4)
+    vals, rows_total, secs_total, cores = [], 0, 0.0, 1
+    for _ in range(args.steps):
+        v, rows, secs, cores = oracle_sample(w, inp, per_step)
+        vals.append(v)
+        rows_total += rows
+        secs_total += secs
+    value = 4.0 * rows_total * w.T * (1 + max(0, min(w.W, w.nodes[0][1] - 1))) * w.d / secs_total / 1e12
+    sample = (f"node {w.nodes[0]} head 0: {rows_total} seeded query rows over {args.steps} steps "
+              f"(fp64 C oracle incl. its RoPE of the node's key states)")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": secs_total / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": config_of(w, world),
+        "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def config_of(w, world):
+    lkv = [w.T * (1 + max(0, min(w.W, b - 1))) for (_, b, _) in w.nodes]
+    return {"workload": w.name, "description": w.description, "nodes": [list(n) for n in w.nodes],
+            "policy": w.policy, "heads": w.H, "head_dim": w.d, "tokens_per_chunk": w.T,
+            "kv_tokens_per_node": lkv, "window_chunks": w.W, "levels": w.K,
+            "l2": "flushed between timed steps (256 MiB write, outside the timed intervals)",
+            "parallelism": "single GPU" if world == 1 else f"{world} independent replicas"}
+
+
+# ---------------------------------------------------------------- GPU arm
+
+def run_ours(args, world, rank, local):
+    import torch
+
+    import __graft_entry__
+    from paper_2609_22283_gb300 import inputs as I
+    from paper_2609_22283_gb300.pipeline import Step
+
+    __graft_entry__.build()
+    if not torch.cuda.is_available():
+        raise RuntimeError("bench.py needs a CUDA GPU (there is no CPU fallback)")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    w = I.WORKLOADS[args.workload]
+    inp = I.generate(w)
+    step = Step(w, device=str(dev))
+    step.prefill(inp)
+    q, k, v = step.device_inputs(inp)
+    out, lse = step.outputs()
+    stream = torch.cuda.current_stream(dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+    nodes, n = step.node_table()
+
+    def one_step():
+        nodes_, _ = step.node_table()            # steps 1-2: selection + Eq. 7 check
+        step.cache.rope_kv_write(nodes_, k, v, q, check=False)
+        step.cache.attend_nodes(nodes_, q, out, lse, step.scale, check=False)
+
+    for _ in range(args.warmup):
+        one_step()
+    status = step.cache.poll()
+    if status != 0:
+        raise RuntimeError(f"device status {status} after warm-up")
+
+    def timed(K):
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+        torch.cuda.synchronize()
+        barrier(world)
+        torch.cuda.synchronize()
+        for i in range(K):
+            flush.zero_()
+            nodes_, _ = step.node_table()
+            ev[i][0].record(stream)
+            step.cache.rope_kv_write(nodes_, k, v, q, check=False)
+            ev[i][1].record(stream)
+            step.cache.attend_nodes(nodes_, q, out, lse, step.scale, check=False)
+            ev[i][2].record(stream)
+        torch.cuda.synchronize()
+        barrier(world)
+        t_rope = sum(e[0].elapsed_time(e[1]) for e in ev)
+        t_attn = sum(e[1].elapsed_time(e[2]) for e in ev)
+        return t_rope, t_attn
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    t_rope, t_attn = timed(args.steps)
+    clocks = sampler.stop()
+    bad = {"hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown"}
+    remeasured = False
+    if clocks and (bad & set(clocks["reasons"])):
+        sampler = ClockSampler(local)
+        sampler.start()
+        time.sleep(0.3)
+        t_rope, t_attn = timed(args.steps)
+        clocks = sampler.stop()
+        remeasured = True
+    status = step.cache.poll()
+    if status != 0:
+        raise RuntimeError(f"device status {status} in the timed region")
+
+    t_step_ms = (t_rope + t_attn) / args.steps
+    t_step_ms = reduce_max(t_step_ms, world)
+    t_attn_ms = reduce_max(t_attn / args.steps, world)
+    t_rope_ms = reduce_max(t_rope / args.steps, world)
+    flops = attn_flops(w)
+    value = flops * world / (t_step_ms * 1e-3) / 1e12
+    nodes_per_s = w.n_nodes * world / (t_step_ms * 1e-3)
+
+    # end to end: host (pinned) inputs -> device, the step, output -> host
+    hq = inp.q.pin_memory()
+    hk = inp.k_new.pin_memory()
+    hv = inp.v_new.pin_memory()
+    hout = torch.empty(out.shape, dtype=out.dtype, pin_memory=True)
+    e2e_ms = []
+    for it in range(args.warmup + min(args.steps, 20)):
+        flush.zero_()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        q.copy_(hq, non_blocking=True)
+        k.copy_(hk, non_blocking=True)
+        v.copy_(hv, non_blocking=True)
+        one_step()
+        hout.copy_(out, non_blocking=True)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if it >= args.warmup:
+            e2e_ms.append(e0.elapsed_time(e1))
+    e2e_step = reduce_max(sum(e2e_ms) / len(e2e_ms), world)
+    h2d = (hq.numel() + hk.numel() + hv.numel()) * 2
+    d2h = hout.numel() * 2
+
+    peaks, peak_src = load_peaks()
+    peak = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
+    achieved = flops / (t_attn_ms * 1e-3) / 1e12
+    traffic = read_traffic(w.name)
+    line = {
+        "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": t_step_ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": config_of(w, world),
+        "nodes_per_s": nodes_per_s,
+        "kernels_ms": {"rope_kv_write": t_rope_ms, "attend_nodes": t_attn_ms},
+        "rope_gbs": rope_bytes(w) / (t_rope_ms * 1e-3) / 1e9,
+        "roofline": {"bound": "tensor", "kernel": "attend_kernel", "achieved": achieved,
+                     "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
+                     "peak_source": f"{peak_src} bf16 dense burst (MEASURED_PEAKS.json)"
+                     if peak_src == "measured" else "fallback 1.9 PFLOP/s",
+                     "traffic": traffic},
+        "e2e": {"value": flops * world / (e2e_step * 1e-3) / 1e12, "unit": "TFLOP/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": 2 * args.steps,
+        "clocks": clocks,
+    }
+    if remeasured:
+        line["clocks_note"] = "first timed region saw a slowdown reason; re-measured once"
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        tf, rows, secs, cores = oracle_sample(w, inp, args.cpu_seconds)
+        line["cpu_baseline"] = {
+            "value": tf, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
+            "sample": f"node {w.nodes[0]} head 0, {rows} seeded query rows, {secs:.1f} s "
+                      f"(fp64 C oracle, OpenMP; incl. its RoPE of the node's key states)"}
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    step.close()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--reference-seconds", type=float, default=8.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        rc = run_reference(args, world, rank)
+    else:
+        rc = run_ours(args, world, rank, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return rc
+
+
+if __name__ == "__main__":
+    sys.exit(main())

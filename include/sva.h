@@ -194,6 +194,17 @@ sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes
  * CUDA if the stream reported an error, else OK. */
 sva_status sva_poll_device_status(sva_cache* c, sva_stream s);
 
+/* Test hook for failure detection; no GPU fault is involved.  mode 1 makes
+ * the next sva_attend_nodes launch on `c` withhold one of its V-tile copies,
+ * so the kernel's bounded wait on that copy expires after timeout_s; every
+ * CTA then records SVA_ERR_DEVICE_TIMEOUT in the status word, waits for its
+ * own copies and MMAs in flight, frees its tensor memory and exits, and
+ * sva_poll_device_status reports the timeout.  Needs nodes of >= 2 key
+ * tiles.  mode 0 clears the hook.  timeout_s (1 ms .. 60 s) also becomes the
+ * bounded-wait limit of this cache's later launches (default 1 s).
+ * Errors: INVALID_ARGUMENT. */
+sva_status sva_debug_inject(sva_cache* c, int32_t mode, double timeout_s);
+
 /* Frees the cache object (not the caller's device buffer). */
 sva_status sva_destroy(sva_cache* c);
 

@@ -1,0 +1,71 @@
+// Parameter blocks passed from the host runtime (sva_api.cpp) to the two
+// kernels, by value as __grid_constant__ kernel parameters, so a launch needs
+// no host-to-device copy of its node list.
+#pragma once
+
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "sva.h"
+
+namespace sva {
+
+constexpr int kTile = 128;  // query rows per Q tile and key rows per K/V tile
+constexpr uint64_t kDefaultWaitTimeoutNs = 1000000000ull;  // bounded device waits: 1 s
+
+// Device status word values (a subset of sva_status).
+constexpr int kStatusOk = 0;
+constexpr int kStatusTimeout = SVA_ERR_DEVICE_TIMEOUT;
+
+// One node of an attention launch: its index in q/out/lse and the cache
+// slots it attends, own slot first, then the visible context slots.
+struct AttnNode {
+  int32_t q_index;
+  int32_t n_kv;
+  int32_t slot[1 + SVA_MAX_CTX];
+};
+
+struct alignas(128) AttnParams {
+  CUtensorMap tmap_q;   // q as 4D (d, H, T, n_nodes), box (64, 1, 128, 1), 128B swizzle
+  CUtensorMap tmap_kv;  // slot pool as 2D (d, num_slots*2*H*Tpad), box (64, 128), 128B swizzle
+  void* out;            // bf16 [n_nodes][T][H][d]
+  float* lse;           // fp32 [n_nodes][H][T] or null
+  int* status;          // device status word
+  float scale_log2;     // logit scale * log2(e)
+  int32_t T;            // tokens per chunk
+  int32_t Tpad;         // T rounded up to kTile: rows per (slot, K|V, head)
+  int32_t H;
+  int32_t n_qt;         // query tiles per node = ceil(T / kTile)
+  int32_t n_nodes;
+  int32_t nt_slot;      // key tiles per slot = Tpad / kTile
+  int32_t valid_last;   // valid key rows in the last tile of a slot
+  int32_t fault_mode;   // 0 in production; see sva_api.cpp
+  uint64_t timeout_ns;
+  AttnNode nodes[SVA_MAX_NODES];
+};
+
+struct RopeNode {
+  int32_t slot;    // own slot the node's K', V go to
+  int32_t t_base;  // absolute latent-frame position of the chunk's first frame (F * chunk)
+};
+
+struct RopeParams {
+  const void* k_new;  // bf16 [n_nodes][T][H][d]
+  const void* v_new;  // bf16 [n_nodes][T][H][d]
+  void* q;            // bf16 [n_nodes][T][H][d], rotated in place; may be null
+  void* cache;        // slot pool base, bf16 [num_slots][2][H][Tpad][d]
+  const float2* tab_t;  // (cos, sin) [max_frames][P0]
+  const float2* tab_h;  // (cos, sin) [Hp][P1]
+  const float2* tab_w;  // (cos, sin) [Wp][P2]
+  int32_t T, H, d, Tpad, Hp, Wp, P0, P1, P2;
+  int32_t n_nodes;
+  int32_t grid_blocks;
+  RopeNode nodes[SVA_MAX_NODES];
+};
+
+// Launchers (defined in the .cu files).  They return the launch error.
+cudaError_t launch_attend(const AttnParams& p, int head_dim, int grid, cudaStream_t s);
+cudaError_t launch_rope_kv(const RopeParams& p, cudaStream_t s);
+
+}  // namespace sva

@@ -1,0 +1,276 @@
+"""ctypes binding of libsva.so (include/sva.h), with the same names.
+
+Argument marshalling only: every step of the hot path runs in the library's
+CUDA kernels.  torch provides device memory and streams; tensors are passed
+as raw device pointers after dtype/shape/contiguity checks.  There is no
+fallback: if libsva.so cannot be loaded, every call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libsva.so")
+
+OK = 0
+ERR_INVALID_ARGUMENT = 1
+ERR_NOT_RESIDENT = 2
+ERR_CAUSALITY = 3
+ERR_CAPACITY = 4
+ERR_UNSUPPORTED = 5
+ERR_CUDA = 6
+ERR_DEVICE_TIMEOUT = 7
+ERR_UNAVAILABLE = 8
+STATUS_NAMES = {0: "OK", 1: "INVALID_ARGUMENT", 2: "NOT_RESIDENT", 3: "CAUSALITY", 4: "CAPACITY",
+                5: "UNSUPPORTED", 6: "CUDA", 7: "DEVICE_TIMEOUT", 8: "UNAVAILABLE"}
+
+POLICY_CLEAN, POLICY_SAME, POLICY_PROG = 0, 1, 2
+POLICIES = {"clean": POLICY_CLEAN, "same": POLICY_SAME, "prog": POLICY_PROG}
+MAX_CTX = 16
+MAX_NODES = 64
+
+EXPORTED = ("sva_cache_bytes", "sva_cache_create", "sva_cache_bind", "sva_cache_lookup",
+            "sva_cache_release", "sva_select_context", "sva_pipeline_round", "sva_check_pipeline",
+            "sva_rope_kv_write", "sva_attend_nodes", "sva_poll_device_status", "sva_debug_inject",
+            "sva_destroy", "sva_last_error")
+
+
+class SvaError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(status, status)}: {message}")
+        self.status = status
+
+
+class sva_geometry(ctypes.Structure):
+    _fields_ = [("num_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("frames", ctypes.c_int32), ("grid_h", ctypes.c_int32), ("grid_w", ctypes.c_int32),
+                ("num_slots", ctypes.c_int32), ("rope_pairs", ctypes.c_int32 * 3),
+                ("max_frames", ctypes.c_int32), ("rope_theta", ctypes.c_double)]
+
+
+class sva_node(ctypes.Structure):
+    _fields_ = [("seq", ctypes.c_int32), ("chunk", ctypes.c_int32), ("level", ctypes.c_int32),
+                ("own_slot", ctypes.c_int32), ("n_ctx", ctypes.c_int32),
+                ("ctx_slot", ctypes.c_int32 * MAX_CTX), ("ctx_visible", ctypes.c_uint8 * MAX_CTX)]
+
+
+_lib = None
+
+
+def load(path: str = LIB_PATH):
+    """Loads libsva.so (built by paper_2609_22283_gb300.build); raises if absent."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with paper_2609_22283_gb300.build.build() "
+                           "(the CUDA library is required; there is no fallback)")
+    lib = ctypes.CDLL(path)
+    i32, p, pi32 = ctypes.c_int32, ctypes.c_void_p, ctypes.POINTER(ctypes.c_int32)
+    pg = ctypes.POINTER(sva_geometry)
+    pn = ctypes.POINTER(sva_node)
+    sig = {
+        "sva_cache_bytes": ([pg], ctypes.c_size_t),
+        "sva_cache_create": ([pg, p, ctypes.c_size_t, ctypes.POINTER(p)], i32),
+        "sva_cache_bind": ([p, i32, i32, i32, pi32], i32),
+        "sva_cache_lookup": ([p, i32, i32, i32, pi32], i32),
+        "sva_cache_release": ([p, i32, i32, i32], i32),
+        "sva_select_context": ([i32, i32, i32, i32, i32, i32, pi32, pi32, pi32], i32),
+        "sva_pipeline_round": ([i32, i32, i32, i32, pi32, pi32, pi32], i32),
+        "sva_check_pipeline": ([i32, i32, i32, i32, pi32, pi32], i32),
+        "sva_rope_kv_write": ([p, pn, i32, p, p, p, p], i32),
+        "sva_attend_nodes": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
+        "sva_poll_device_status": ([p, p], i32),
+        "sva_debug_inject": ([p, i32, ctypes.c_double], i32),
+        "sva_destroy": ([p], i32),
+        "sva_last_error": ([], ctypes.c_char_p),
+    }
+    for name, (args, res) in sig.items():
+        f = getattr(lib, name)
+        f.argtypes = args
+        f.restype = res
+    _lib = lib
+    return lib
+
+
+def _check(status: int):
+    if status != OK:
+        msg = _lib.sva_last_error().decode(errors="replace")
+        raise SvaError(status, msg)
+
+
+def _stream_handle(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream
+
+
+def _tok_major(t: torch.Tensor, name: str, n: int, T: int, H: int, d: int):
+    if t.dtype != torch.bfloat16 or not t.is_cuda or not t.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous bf16 CUDA tensor")
+    if tuple(t.shape) != (n, T, H, d):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, expected {(n, T, H, d)}")
+
+
+# ---------------------------------------------------------------- selection (host)
+
+def select_context(policy: int, K: int, W: int, chunk: int, level: int, cap: int = MAX_CTX):
+    lib = load()
+    ch = (ctypes.c_int32 * max(cap, 1))()
+    lv = (ctypes.c_int32 * max(cap, 1))()
+    n = ctypes.c_int32()
+    _check(lib.sva_select_context(policy, K, W, chunk, level, cap, ch, lv, ctypes.byref(n)))
+    return [(ch[i], lv[i]) for i in range(n.value)]
+
+
+def pipeline_round(K: int, B: int, n: int, cap: int = 64):
+    lib = load()
+    ch = (ctypes.c_int32 * cap)()
+    lv = (ctypes.c_int32 * cap)()
+    cnt = ctypes.c_int32()
+    _check(lib.sva_pipeline_round(K, B, n, cap, ch, lv, ctypes.byref(cnt)))
+    return [(ch[i], lv[i]) for i in range(cnt.value)]
+
+
+def check_pipeline(K: int, level: int, chunk: int, states) -> int:
+    """Returns the sva_status of the Eq. 7 check (no exception for UNAVAILABLE)."""
+    lib = load()
+    n = len(states)
+    ch = (ctypes.c_int32 * max(n, 1))(*[c for c, _ in states])
+    lv = (ctypes.c_int32 * max(n, 1))(*[l for _, l in states])
+    return int(lib.sva_check_pipeline(K, level, chunk, n, ch, lv))
+
+
+def last_error() -> str:
+    return load().sva_last_error().decode(errors="replace")
+
+
+def make_geometry(H, d, F, Hp, Wp, num_slots, pairs, max_frames, theta=10000.0) -> sva_geometry:
+    g = sva_geometry()
+    g.num_heads, g.head_dim, g.frames, g.grid_h, g.grid_w = H, d, F, Hp, Wp
+    g.num_slots = num_slots
+    g.rope_pairs[0], g.rope_pairs[1], g.rope_pairs[2] = pairs
+    g.max_frames = max_frames
+    g.rope_theta = theta
+    return g
+
+
+def cache_bytes(g: sva_geometry) -> int:
+    return int(load().sva_cache_bytes(ctypes.byref(g)))
+
+
+def make_nodes(entries) -> ctypes.Array:
+    """entries: iterable of dicts with seq, chunk, level, own_slot, ctx (list of slots),
+    visible (optional list of 0/1)."""
+    entries = list(entries)
+    arr = (sva_node * max(len(entries), 1))()
+    for i, e in enumerate(entries):
+        n = arr[i]
+        n.seq, n.chunk, n.level, n.own_slot = e["seq"], e["chunk"], e["level"], e["own_slot"]
+        ctx = list(e.get("ctx", []))
+        vis = list(e.get("visible", [1] * len(ctx)))
+        n.n_ctx = len(ctx)
+        for k, s in enumerate(ctx[:MAX_CTX]):
+            n.ctx_slot[k] = s
+            n.ctx_visible[k] = vis[k]
+    return arr
+
+
+class Cache:
+    """A KV cache over a caller-owned device buffer (a torch uint8 tensor)."""
+
+    def __init__(self, g: sva_geometry, buf: torch.Tensor | None = None, device=None):
+        lib = load()
+        self.g = g
+        self.nbytes = cache_bytes(g)
+        if self.nbytes == 0:
+            raise SvaError(ERR_INVALID_ARGUMENT, last_error())
+        if buf is None:
+            buf = torch.empty(self.nbytes, dtype=torch.uint8, device=device or "cuda")
+        if not buf.is_cuda or buf.numel() * buf.element_size() < self.nbytes:
+            raise ValueError("cache buffer must be a CUDA tensor of at least cache_bytes(g) bytes")
+        self.buf = buf
+        self.T = g.frames * g.grid_h * g.grid_w
+        self.Tpad = (self.T + 127) // 128 * 128
+        handle = ctypes.c_void_p()
+        with torch.cuda.device(buf.device):
+            _check(lib.sva_cache_create(ctypes.byref(g), ctypes.c_void_p(buf.data_ptr()),
+                                        self.nbytes, ctypes.byref(handle)))
+        self.handle = handle
+
+    # slot pool view [num_slots][2][H][Tpad][d] (bf16), for inspection in tests
+    def slot_pool(self) -> torch.Tensor:
+        g = self.g
+        n = g.num_slots * 2 * g.num_heads * self.Tpad * g.head_dim
+        return self.buf[: n * 2].view(torch.bfloat16).view(g.num_slots, 2, g.num_heads, self.Tpad,
+                                                           g.head_dim)
+
+    def bind(self, seq: int, chunk: int, level: int) -> int:
+        s = ctypes.c_int32()
+        _check(_lib.sva_cache_bind(self.handle, seq, chunk, level, ctypes.byref(s)))
+        return s.value
+
+    def lookup(self, seq: int, chunk: int, level: int) -> int:
+        s = ctypes.c_int32()
+        _check(_lib.sva_cache_lookup(self.handle, seq, chunk, level, ctypes.byref(s)))
+        return s.value
+
+    def release(self, seq: int, chunk: int, level: int):
+        _check(_lib.sva_cache_release(self.handle, seq, chunk, level))
+
+    def rope_kv_write(self, nodes, k_new, v_new, q=None, stream=None, check=True):
+        n = len(nodes) if not isinstance(nodes, ctypes.Array) else None
+        arr = nodes if isinstance(nodes, ctypes.Array) else make_nodes(nodes)
+        count = n if n is not None else len(arr)
+        if check:
+            g = self.g
+            _tok_major(k_new, "k_new", count, self.T, g.num_heads, g.head_dim)
+            _tok_major(v_new, "v_new", count, self.T, g.num_heads, g.head_dim)
+            if q is not None:
+                _tok_major(q, "q", count, self.T, g.num_heads, g.head_dim)
+        st = _lib.sva_rope_kv_write(self.handle, arr, count, ctypes.c_void_p(k_new.data_ptr()),
+                                    ctypes.c_void_p(v_new.data_ptr()),
+                                    ctypes.c_void_p(q.data_ptr() if q is not None else 0),
+                                    ctypes.c_void_p(_stream_handle(stream)))
+        _check(st)
+
+    def attend_nodes(self, nodes, q, out, lse=None, scale=None, stream=None, check=True):
+        n = len(nodes) if not isinstance(nodes, ctypes.Array) else None
+        arr = nodes if isinstance(nodes, ctypes.Array) else make_nodes(nodes)
+        count = n if n is not None else len(arr)
+        g = self.g
+        if check:
+            _tok_major(q, "q", count, self.T, g.num_heads, g.head_dim)
+            _tok_major(out, "out", count, self.T, g.num_heads, g.head_dim)
+            if lse is not None and (lse.dtype != torch.float32 or not lse.is_contiguous()
+                                    or tuple(lse.shape) != (count, g.num_heads, self.T)):
+                raise ValueError("lse must be a contiguous fp32 tensor [n][H][T]")
+        if scale is None:
+            scale = 1.0 / math.sqrt(g.head_dim)
+        st = _lib.sva_attend_nodes(self.handle, arr, count, ctypes.c_void_p(q.data_ptr()),
+                                   ctypes.c_void_p(out.data_ptr()),
+                                   ctypes.c_void_p(lse.data_ptr() if lse is not None else 0),
+                                   float(scale), ctypes.c_void_p(_stream_handle(stream)))
+        _check(st)
+
+    def poll(self, stream=None) -> int:
+        """sva_poll_device_status: returns the status code (0 = OK)."""
+        return int(_lib.sva_poll_device_status(self.handle, ctypes.c_void_p(_stream_handle(stream))))
+
+    def debug_inject(self, mode: int, timeout_s: float = 1.0):
+        _check(_lib.sva_debug_inject(self.handle, mode, float(timeout_s)))
+
+    def close(self):
+        if getattr(self, "handle", None):
+            _lib.sva_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -17,3 +17,11 @@ def oracle_mod():
     import oracle
     oracle.build()
     return oracle
+
+
+@pytest.fixture(scope="session")
+def sva_mod():
+    from paper_2609_22283_gb300 import build, sva
+    build.build()
+    sva.load()
+    return sva
