@@ -8,17 +8,22 @@
 // outside those slots are never read, so the mask costs nothing except on the
 // zero pad rows of each slot's last tile, which get -inf explicitly.
 //
-// One CTA computes one work unit (node, head, 128-query tile) and streams
-// every key tile of every slot the node reads:
-//   warp 0    TMA producer: Q once, then K and V tiles of the slot list into
-//             a ring of shared-memory stages (128B swizzle);
-//   warp 1    MMA issuer (one thread): S = Q K^T into one of two TMEM
-//             buffers, then O += P V with P read from TMEM;
-//   warps 2-5 softmax: one query row per thread; S from TMEM, fp32 online
-//             softmax in the log2 domain with a lazy rescale of O, P written
-//             back into the S buffer as bf16; then the epilogue (O / l to
-//             bf16 global, optional LSE).
-// TMEM columns: S0 [0,128), S1 [128,256), O [256, 256+d).
+// One CTA computes one work unit: (node, head, a pair of 128-query tiles Q0,
+// Q1) and streams every key tile of every slot the node reads; each K/V tile
+// in shared memory serves both query tiles.
+//   warp 0     TMA producer: Q0/Q1 once, then K and V tiles of the slot list
+//              into rings of shared-memory stages (128B swizzle);
+//   warp 1     MMA issuer (one thread) and TMEM owner;
+//   warps 2-5  softmax of Q0, warps 6-9 softmax of Q1: one query row per
+//              thread; S from TMEM, fp32 online softmax in the log2 domain
+//              with a lazy rescale of O, P written back over S as bf16; then
+//              the epilogue (O / l to bf16 global, optional LSE).
+// TMEM columns: S0 [0,128), S1 [128,256), O0 [256, 256+d), O1 [384, 384+d).
+// MMA order per key tile i: PV0_i, S0_{i+1}, PV1_i, S1_{i+1}, so either
+// softmax warpgroup has the other tile's PV and S (two 128x128x128 MMAs) to
+// hide behind.  A commit that completes S_b of tile i also implies PV_b of
+// tile i-1 is complete (MMAs execute in issue order), so the rescale of O_b
+// needs no extra barrier.
 // All waits are bounded (1 s by default): on expiry the CTA records
 // SVA_ERR_DEVICE_TIMEOUT in the status word, drains its own copies and MMAs,
 // frees TMEM and exits.
@@ -39,23 +44,57 @@ struct AttnCfg {
   static constexpr int kBoxBytes = kTile * 64 * 2;   // one 128-row x 64-column bf16 box
   static constexpr int kBoxes = D / 64;
   static constexpr int kTileBytes = kBoxBytes * kBoxes;
-  static constexpr int kStages = (D == 128) ? 3 : 4;
-  static constexpr int kOffQ = 0;
-  static constexpr int kOffK = kOffQ + kTileBytes;
-  static constexpr int kOffV = kOffK + kStages * kTileBytes;
-  static constexpr int kSmemBytes = kOffV + kStages * kTileBytes + 1024;  // + alignment slack
-  static constexpr uint32_t kColS = 0;      // S buffers at columns 0 and 128
-  static constexpr uint32_t kColO = 256;
+  static constexpr int kKStages = (D == 128) ? 3 : 4;
+  static constexpr int kVStages = (D == 128) ? 2 : 4;
+  static constexpr int kOffQ0 = 0;
+  static constexpr int kOffQ1 = kTileBytes;
+  static constexpr int kOffK = 2 * kTileBytes;
+  static constexpr int kOffV = kOffK + kKStages * kTileBytes;
+  static constexpr int kSmemBytes = kOffV + kVStages * kTileBytes + 1024;  // + alignment slack
   static constexpr uint32_t kTmemCols = 512;
 };
 
-constexpr int kThreads = 192;
+// TMEM columns of the S buffers and O accumulators of query tiles 0 and 1.
+__device__ __forceinline__ uint32_t col_s(int b) { return b ? 128u : 0u; }
+__device__ __forceinline__ uint32_t col_o(int b) { return b ? 384u : 256u; }
+
+constexpr int kThreads = 320;
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: P <= 2^8 between rescales
 
 __device__ __forceinline__ float ex2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+__device__ __forceinline__ uint64_t f2u(float a, float b) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+  return r;
+}
+
+__device__ __forceinline__ void u2f(uint64_t r, float& a, float& b) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(r));
+}
+
+// (a0, a1) * bb + cc, two lanes in one instruction
+__device__ __forceinline__ void ffma2(float& o0, float& o1, float a0, float a1, uint64_t bb,
+                                      uint64_t cc) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(f2u(a0, a1)), "l"(bb), "l"(cc));
+  u2f(r, o0, o1);
+}
+
+__device__ __forceinline__ uint64_t fadd2(uint64_t a, float b0, float b1) {
+  uint64_t r;
+  asm("add.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(f2u(b0, b1)));
+  return r;
 }
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
@@ -67,7 +106,6 @@ struct Bars {
   uint64_t q_full;
   uint64_t s_full[2];
   uint64_t p_full[2];
-  uint64_t o_ready;
   uint64_t o_final;
   uint64_t drain;
   uint64_t k_full[4];
@@ -96,26 +134,29 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
 
   // Work unit, head-major so the CTAs that share a head's K/V run together.
   const int unit = blockIdx.x;
-  const int qt = unit % p.n_qt;
-  const int rest = unit / p.n_qt;
+  const int qp = unit % p.n_qp;
+  const int rest = unit / p.n_qp;
   const int ni = rest % p.n_nodes;
   const int h = rest / p.n_nodes;
   const AttnNode& nd = p.nodes[ni];
   const int n_tiles = nd.n_kv * p.nt_slot;
+  const int qt0 = 2 * qp;
+  const bool has_q1 = qt0 + 1 < p.n_qt;
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
     mbar_init(&bars.q_full, 1);
-    mbar_init(&bars.o_ready, 1);
     mbar_init(&bars.o_final, 1);
     mbar_init(&bars.drain, 1);
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bars.s_full[b], 1);
       mbar_init(&bars.p_full[b], 128);
     }
-    for (int s = 0; s < C::kStages; ++s) {
+    for (int s = 0; s < C::kKStages; ++s) {
       mbar_init(&bars.k_full[s], 1);
       mbar_init(&bars.k_empty[s], 1);
+    }
+    for (int s = 0; s < C::kVStages; ++s) {
       mbar_init(&bars.v_full[s], 1);
       mbar_init(&bars.v_empty[s], 1);
     }
@@ -131,7 +172,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
   const uint32_t tbase = tmem_base_sh;
   const uint64_t tmo = p.timeout_ns;
 
-  uint8_t* sQ = smem + C::kOffQ;
+  uint8_t* sQ0 = smem + C::kOffQ0;
+  uint8_t* sQ1 = smem + C::kOffQ1;
   uint8_t* sK = smem + C::kOffK;
   uint8_t* sV = smem + C::kOffV;
   int k_issued = 0, v_issued = 0;  // producer: tiles whose K / V copies were started
@@ -141,41 +183,47 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     if (lane == 0) {
       prefetch_tmap(&p.tmap_q);
       prefetch_tmap(&p.tmap_kv);
-      mbar_arrive_expect_tx(&bars.q_full, C::kTileBytes);
+      mbar_arrive_expect_tx(&bars.q_full, (has_q1 ? 2 : 1) * C::kTileBytes);
 #pragma unroll
-      for (int b = 0; b < C::kBoxes; ++b)
-        tma_load_4d(sQ + b * C::kBoxBytes, &p.tmap_q, &bars.q_full, b * 64, h, qt * kTile,
+      for (int b = 0; b < C::kBoxes; ++b) {
+        tma_load_4d(sQ0 + b * C::kBoxBytes, &p.tmap_q, &bars.q_full, b * 64, h, qt0 * kTile,
                     nd.q_index);
+        if (has_q1)
+          tma_load_4d(sQ1 + b * C::kBoxBytes, &p.tmap_q, &bars.q_full, b * 64, h,
+                      (qt0 + 1) * kTile, nd.q_index);
+      }
       const uint64_t keep = l2_policy_evict_last();
       for (int i = 0; i < n_tiles; ++i) {
-        const int st = i % C::kStages;
-        const uint32_t ph = (uint32_t)(i / C::kStages) & 1u;
+        const int ks = i % C::kKStages;
+        const int vs = i % C::kVStages;
         const int slot = nd.slot[i / p.nt_slot];
         const int t = i - (i / p.nt_slot) * p.nt_slot;
         const int row_k = ((slot * 2 + 0) * p.H + h) * p.Tpad + t * kTile;
         const int row_v = row_k + p.H * p.Tpad;
-        if (!mbar_wait(&bars.k_empty[st], ph ^ 1u, &abort_flag, tmo)) {
+        if (!mbar_wait(&bars.k_empty[ks], ((uint32_t)(i / C::kKStages) & 1u) ^ 1u, &abort_flag,
+                       tmo)) {
           record_timeout(p, &abort_flag);
           break;
         }
-        mbar_arrive_expect_tx(&bars.k_full[st], C::kTileBytes);
+        mbar_arrive_expect_tx(&bars.k_full[ks], C::kTileBytes);
 #pragma unroll
         for (int b = 0; b < C::kBoxes; ++b)
-          tma_load_2d_hint(sK + st * C::kTileBytes + b * C::kBoxBytes, &p.tmap_kv,
-                           &bars.k_full[st], b * 64, row_k, keep);
+          tma_load_2d_hint(sK + ks * C::kTileBytes + b * C::kBoxBytes, &p.tmap_kv,
+                           &bars.k_full[ks], b * 64, row_k, keep);
         k_issued = i + 1;
-        if (!mbar_wait(&bars.v_empty[st], ph ^ 1u, &abort_flag, tmo)) {
+        if (!mbar_wait(&bars.v_empty[vs], ((uint32_t)(i / C::kVStages) & 1u) ^ 1u, &abort_flag,
+                       tmo)) {
           record_timeout(p, &abort_flag);
           break;
         }
         // fault_mode 1 (test hook): withhold the V copy of tile 1, so the
         // MMA issuer's bounded wait on it expires.
         if (!(p.fault_mode == 1 && i == 1)) {
-          mbar_arrive_expect_tx(&bars.v_full[st], C::kTileBytes);
+          mbar_arrive_expect_tx(&bars.v_full[vs], C::kTileBytes);
 #pragma unroll
           for (int b = 0; b < C::kBoxes; ++b)
-            tma_load_2d_hint(sV + st * C::kTileBytes + b * C::kBoxBytes, &p.tmap_kv,
-                             &bars.v_full[st], b * 64, row_v, keep);
+            tma_load_2d_hint(sV + vs * C::kTileBytes + b * C::kBoxBytes, &p.tmap_kv,
+                             &bars.v_full[vs], b * 64, row_v, keep);
         }
         v_issued = i + 1;
       }
@@ -185,51 +233,74 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     if (lane == 0) {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(128, 128, false);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, true);
-      const uint32_t aQ = smem_u32(sQ);
+      const uint32_t aQ0 = smem_u32(sQ0);
+      const uint32_t aQ1 = smem_u32(sQ1);
       const uint32_t aK = smem_u32(sK);
       const uint32_t aV = smem_u32(sV);
-      bool ok = mbar_wait(&bars.q_full, 0, &abort_flag, tmo);
-      tc_fence_after();
-      auto issue_qk = [&](int i) -> bool {
-        const int st = i % C::kStages;
-        const uint32_t ph = (uint32_t)(i / C::kStages) & 1u;
-        if (!mbar_wait(&bars.k_full[st], ph, &abort_flag, tmo)) return false;
-        tc_fence_after();
-        const uint32_t dcol = tbase + C::kColS + (uint32_t)(i & 1) * 128u;
-        const uint32_t kb = aK + st * C::kTileBytes;
+      // S_b = Q_b K_i^T into TMEM buffer b
+      auto issue_s = [&](int b, int i) {
+        const uint32_t kb = aK + (i % C::kKStages) * C::kTileBytes;
+        const uint32_t qb = b ? aQ1 : aQ0;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t off = (kk >> 2) * C::kBoxBytes + (kk & 3) * 32;
-          mma_ss(dcol, sdesc_sw128(aQ + off, 16, 1024), sdesc_sw128(kb + off, 16, 1024), idesc_qk,
-                 kk > 0 ? 1u : 0u);
+          mma_ss(tbase + col_s(b), sdesc_sw128(qb + off, 16, 1024),
+                 sdesc_sw128(kb + off, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
         }
-        mma_commit(&bars.k_empty[st]);
-        mma_commit(&bars.s_full[i & 1]);
-        return true;
+        mma_commit(&bars.s_full[b]);
       };
-      if (ok) ok = issue_qk(0);
+      // O_b += P_b V_i with P_b read from TMEM over S_b
+      auto issue_pv = [&](int b, int i) {
+        const uint32_t vb = aV + (i % C::kVStages) * C::kTileBytes;
+#pragma unroll
+        for (int kk = 0; kk < kTile / 16; ++kk)
+          mma_ts(tbase + col_o(b), tbase + col_s(b) + kk * 8,
+                 sdesc_sw128(vb + kk * 2048, C::kBoxBytes, 1024), idesc_pv,
+                 (i > 0 || kk > 0) ? 1u : 0u);
+      };
+      auto wait_k = [&](int i) {
+        return mbar_wait(&bars.k_full[i % C::kKStages], (uint32_t)(i / C::kKStages) & 1u,
+                         &abort_flag, tmo);
+      };
+      bool ok = mbar_wait(&bars.q_full, 0, &abort_flag, tmo) && wait_k(0);
+      if (ok) {
+        tc_fence_after();
+        issue_s(0, 0);
+        if (has_q1) issue_s(1, 0);
+        mma_commit(&bars.k_empty[0]);
+      }
       for (int i = 0; ok && i < n_tiles; ++i) {
-        if (i + 1 < n_tiles && !issue_qk(i + 1)) {
-          ok = false;
-          break;
-        }
-        const int st = i % C::kStages;
-        const uint32_t ph = (uint32_t)(i / C::kStages) & 1u;
-        if (!mbar_wait(&bars.p_full[i & 1], (uint32_t)(i >> 1) & 1u, &abort_flag, tmo) ||
-            !mbar_wait(&bars.v_full[st], ph, &abort_flag, tmo)) {
+        const uint32_t par = (uint32_t)i & 1u;
+        if (!mbar_wait(&bars.p_full[0], par, &abort_flag, tmo) ||
+            !mbar_wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u,
+                       &abort_flag, tmo)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t pcol = tbase + C::kColS + (uint32_t)(i & 1) * 128u;
-        const uint32_t vb = aV + st * C::kTileBytes;
-#pragma unroll
-        for (int kk = 0; kk < kTile / 16; ++kk) {
-          mma_ts(tbase + C::kColO, pcol + kk * 8, sdesc_sw128(vb + kk * 2048, C::kBoxBytes, 1024),
-                 idesc_pv, (i > 0 || kk > 0) ? 1u : 0u);
+        issue_pv(0, i);
+        const bool more = i + 1 < n_tiles;
+        if (more) {
+          if (!wait_k(i + 1)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          issue_s(0, i + 1);
         }
-        mma_commit(&bars.v_empty[st]);
-        mma_commit(&bars.o_ready);
+        if (has_q1) {
+          if (!mbar_wait(&bars.p_full[1], par, &abort_flag, tmo)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          issue_pv(1, i);
+        }
+        mma_commit(&bars.v_empty[i % C::kVStages]);
+        if (more) {
+          if (has_q1) issue_s(1, i + 1);
+          mma_commit(&bars.k_empty[(i + 1) % C::kKStages]);
+        }
       }
       if (ok) {
         mma_commit(&bars.o_final);
@@ -239,121 +310,154 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     }
   } else {
     // ------------------------------------------------------------ softmax + epilogue
+    const int b = (warp - 2) >> 2;                 // query tile of this warpgroup
     const int q4 = warp & 3;                       // TMEM lane quarter this warp may access
     const int row = q4 * 32 + lane;                // query row inside the tile
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
-    const float sl2 = p.scale_log2;
-    float m = -INFINITY;  // running max of scale*log2(e)*logit (possibly stale by < threshold)
-    float l = 0.0f;       // running sum of 2^(x - m)
-    bool ok = true;
-    for (int i = 0; i < n_tiles; ++i) {
-      const int buf = i & 1;
-      ok = mbar_wait(&bars.s_full[buf], (uint32_t)(i >> 1) & 1u, &abort_flag, tmo);
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok) break;
-      tc_fence_after();
-      const uint32_t scol = tbase + lane_off + C::kColS + (uint32_t)buf * 128u;
-      uint32_t s[4][32];
+    if (b == 0 || has_q1) {
+      const float sl2 = p.scale_log2;
+      const uint64_t sl2x2 = f2u(sl2, sl2);
+      const uint32_t scol = tbase + lane_off + col_s(b);
+      const uint32_t ocol = tbase + lane_off + col_o(b);
+      float m = -INFINITY;  // running max of scale*log2(e)*logit (possibly stale by < threshold)
+      float l = 0.0f;       // running sum of 2^(x - m)
+      bool ok = true;
+      for (int i = 0; i < n_tiles; ++i) {
+        ok = mbar_wait(&bars.s_full[b], (uint32_t)i & 1u, &abort_flag, tmo);
+        ok = __all_sync(0xffffffffu, ok);
+        if (!ok) break;
+        tc_fence_after();
+        const int t = i % p.nt_slot;
+        const int valid = (t == p.nt_slot - 1) ? p.valid_last : kTile;
+        float m_tile;
+        {
+          // pass 1: row max over the 128 keys of the tile
+          uint32_t s[4][32];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_ld32(scol + c * 32, s[c]);
+          for (int c = 0; c < 4; ++c) tmem_ld32(scol + c * 32, s[c]);
 #pragma unroll
-      for (int c = 0; c < 4; ++c) tmem_wait_ld(s[c]);
-
-      const int t = i % p.nt_slot;
-      const int valid = (t == p.nt_slot - 1) ? p.valid_last : kTile;
-      if (valid < kTile) {
+          for (int c = 0; c < 4; ++c) tmem_wait_ld(s[c]);
+          if (valid < kTile) {
 #pragma unroll
-        for (int c = 0; c < 4; ++c)
+            for (int c = 0; c < 4; ++c)
 #pragma unroll
-          for (int e = 0; e < 32; ++e)
-            if (c * 32 + e >= valid) s[c][e] = __float_as_uint(-INFINITY);
-      }
-      float mx0 = -INFINITY, mx1 = -INFINITY, mx2 = -INFINITY, mx3 = -INFINITY;
-#pragma unroll
-      for (int e = 0; e < 32; ++e) {
-        mx0 = fmaxf(mx0, __uint_as_float(s[0][e]));
-        mx1 = fmaxf(mx1, __uint_as_float(s[1][e]));
-        mx2 = fmaxf(mx2, __uint_as_float(s[2][e]));
-        mx3 = fmaxf(mx3, __uint_as_float(s[3][e]));
-      }
-      const float m_tile = fmaxf(fmaxf(mx0, mx1), fmaxf(mx2, mx3)) * sl2;
-      const float m_new = fmaxf(m, m_tile);
-      const bool need = m_new > m + kRescaleThreshold;
-      if (__any_sync(0xffffffffu, need)) {
-        const float alpha = ex2(m - m_new);  // 0 on the first tile (m = -inf)
-        if (i > 0) {
-          // O holds the sum over tiles < i once PV_{i-1} is complete.
-          ok = mbar_wait(&bars.o_ready, (uint32_t)(i - 1) & 1u, &abort_flag, tmo);
-          ok = __all_sync(0xffffffffu, ok);
-          if (!ok) break;
-          tc_fence_after();
-#pragma unroll
-          for (int c = 0; c < D / 32; ++c) {
-            uint32_t o[32];
-            const uint32_t ocol = tbase + lane_off + C::kColO + c * 32;
-            tmem_ld32(ocol, o);
-            tmem_wait_ld(o);
-#pragma unroll
-            for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-            tmem_st32(ocol, o);
+              for (int e = 0; e < 32; ++e)
+                if (c * 32 + e >= valid) s[c][e] = __float_as_uint(-INFINITY);
           }
-          tmem_wait_st();
+          float mx[8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k) mx[k] = -INFINITY;
+#pragma unroll
+          for (int c = 0; c < 4; ++c)
+#pragma unroll
+            for (int e = 0; e < 32; e += 8) {
+              const int k = (c & 1) * 4 + (e >> 3);
+              mx[k] = max3(mx[k], __uint_as_float(s[c][e]), __uint_as_float(s[c][e + 1]));
+              mx[k] = max3(mx[k], __uint_as_float(s[c][e + 2]), __uint_as_float(s[c][e + 3]));
+              mx[k] = max3(mx[k], __uint_as_float(s[c][e + 4]), __uint_as_float(s[c][e + 5]));
+              mx[k] = max3(mx[k], __uint_as_float(s[c][e + 6]), __uint_as_float(s[c][e + 7]));
+            }
+          m_tile = max3(max3(mx[0], mx[1], mx[2]), max3(mx[3], mx[4], mx[5]),
+                        fmaxf(mx[6], mx[7])) * sl2;
         }
-        l *= alpha;
-        m = m_new;
+        const float m_new = fmaxf(m, m_tile);
+        const bool need = m_new > m + kRescaleThreshold;
+        if (__any_sync(0xffffffffu, need)) {
+          const float alpha = ex2(m - m_new);  // 0 on the first tile (m = -inf)
+          if (i > 0) {
+            // O_b holds the sum over tiles < i: the commit that completed S_b
+            // of tile i came after PV_b of tile i-1.
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+              uint32_t o[32];
+              tmem_ld32(ocol + c * 32, o);
+              tmem_wait_ld(o);
+#pragma unroll
+              for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
+              tmem_st32(ocol + c * 32, o);
+            }
+            tmem_wait_st();
+          }
+          l *= alpha;
+          m = m_new;
+        }
+        const uint64_t negm = f2u(-m, -m);
+        uint64_t acc[4] = {0, 0, 0, 0};
+        // pass 2: S again, 64 keys at a time; P of 32 keys packs into 16
+        // words written over the first half of the same registers (word e/2
+        // is written after elements e, e+1 are read), then stored over S.
+#pragma unroll
+        for (int c2 = 0; c2 < 2; ++c2) {
+          uint32_t s[2][32];
+          tmem_ld32(scol + c2 * 64, s[0]);
+          tmem_ld32(scol + c2 * 64 + 32, s[1]);
+          tmem_wait_ld(s[0]);
+          tmem_wait_ld(s[1]);
+          if (valid < kTile) {
+#pragma unroll
+            for (int cc = 0; cc < 2; ++cc)
+#pragma unroll
+              for (int e = 0; e < 32; ++e)
+                if (c2 * 64 + cc * 32 + e >= valid) s[cc][e] = __float_as_uint(-INFINITY);
+          }
+#pragma unroll
+          for (int cc = 0; cc < 2; ++cc)
+#pragma unroll
+            for (int e = 0; e < 32; e += 2) {
+              float x0, x1;
+              ffma2(x0, x1, __uint_as_float(s[cc][e]), __uint_as_float(s[cc][e + 1]), sl2x2, negm);
+              const float p0 = ex2(x0);
+              const float p1 = ex2(x1);
+              acc[(e >> 1) & 3] = fadd2(acc[(e >> 1) & 3], p0, p1);
+              s[cc][e >> 1] = pack_bf16(p0, p1);
+            }
+          tmem_st32_halves(scol + c2 * 32, s[0], s[1]);
+        }
+        float a0, a1, a2, a3, a4, a5, a6, a7;
+        u2f(acc[0], a0, a1);
+        u2f(acc[1], a2, a3);
+        u2f(acc[2], a4, a5);
+        u2f(acc[3], a6, a7);
+        l += ((a0 + a1) + (a2 + a3)) + ((a4 + a5) + (a6 + a7));
+        tmem_wait_st();
+        tc_fence_before();
+        mbar_arrive(&bars.p_full[b]);
       }
-      float sum0 = 0.f, sum1 = 0.f;
-      uint32_t pk[2][32];
+      if (ok) {
+        ok = mbar_wait(&bars.o_final, 0, &abort_flag, tmo);
+        ok = __all_sync(0xffffffffu, ok);
+      }
+      if (!ok) {
+        record_timeout(p, &abort_flag);
+      } else {
+        tc_fence_after();
+        const int token = (qt0 + b) * kTile + row;
+        const bool in_range = token < p.T;
+        const float inv_l = 1.0f / l;
+        __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(p.out) +
+                              (((size_t)nd.q_index * p.T + token) * p.H + h) * D;
 #pragma unroll
-      for (int c = 0; c < 4; ++c)
+        for (int c = 0; c < D / 32; ++c) {
+          uint32_t o[32];
+          tmem_ld32(ocol + c * 32, o);
+          tmem_wait_ld(o);
+          if (in_range) {
+            uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
 #pragma unroll
-        for (int e = 0; e < 32; e += 2) {
-          const float p0 = ex2(fmaf(__uint_as_float(s[c][e]), sl2, -m));
-          const float p1 = ex2(fmaf(__uint_as_float(s[c][e + 1]), sl2, -m));
-          sum0 += p0;
-          sum1 += p1;
-          pk[c >> 1][(c & 1) * 16 + (e >> 1)] = pack_bf16(p0, p1);
-        }
-      l += sum0 + sum1;
-      tmem_st32(scol, pk[0]);
-      tmem_st32(scol + 32, pk[1]);
-      tmem_wait_st();
-      tc_fence_before();
-      mbar_arrive(&bars.p_full[buf]);
-    }
-    if (ok) {
-      ok = mbar_wait(&bars.o_final, 0, &abort_flag, tmo);
-      ok = __all_sync(0xffffffffu, ok);
-    }
-    if (!ok) {
-      record_timeout(p, &abort_flag);
-    } else {
-      tc_fence_after();
-      const int token = qt * kTile + row;
-      const bool in_range = token < p.T;
-      const float inv_l = 1.0f / l;
-      __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(p.out) +
-                            (((size_t)nd.q_index * p.T + token) * p.H + h) * D;
-#pragma unroll
-      for (int c = 0; c < D / 32; ++c) {
-        uint32_t o[32];
-        tmem_ld32(tbase + lane_off + C::kColO + c * 32, o);
-        tmem_wait_ld(o);
-        if (in_range) {
-          uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
-#pragma unroll
-          for (int v = 0; v < 4; ++v) {
-            uint4 w;
-            w.x = pack_bf16(__uint_as_float(o[v * 8 + 0]) * inv_l, __uint_as_float(o[v * 8 + 1]) * inv_l);
-            w.y = pack_bf16(__uint_as_float(o[v * 8 + 2]) * inv_l, __uint_as_float(o[v * 8 + 3]) * inv_l);
-            w.z = pack_bf16(__uint_as_float(o[v * 8 + 4]) * inv_l, __uint_as_float(o[v * 8 + 5]) * inv_l);
-            w.w = pack_bf16(__uint_as_float(o[v * 8 + 6]) * inv_l, __uint_as_float(o[v * 8 + 7]) * inv_l);
-            dst[v] = w;
+            for (int v = 0; v < 4; ++v) {
+              uint4 w;
+              w.x = pack_bf16(__uint_as_float(o[v * 8 + 0]) * inv_l, __uint_as_float(o[v * 8 + 1]) * inv_l);
+              w.y = pack_bf16(__uint_as_float(o[v * 8 + 2]) * inv_l, __uint_as_float(o[v * 8 + 3]) * inv_l);
+              w.z = pack_bf16(__uint_as_float(o[v * 8 + 4]) * inv_l, __uint_as_float(o[v * 8 + 5]) * inv_l);
+              w.w = pack_bf16(__uint_as_float(o[v * 8 + 6]) * inv_l, __uint_as_float(o[v * 8 + 7]) * inv_l);
+              dst[v] = w;
+            }
           }
         }
-      }
-      if (p.lse != nullptr && in_range) {
-        p.lse[((size_t)nd.q_index * p.H + h) * p.T + token] = (m + __log2f(l)) * 0.69314718055994531f;
+        if (p.lse != nullptr && in_range) {
+          p.lse[((size_t)nd.q_index * p.H + h) * p.T + token] =
+              (m + __log2f(l)) * 0.69314718055994531f;
+        }
       }
     }
   }
@@ -370,11 +474,11 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     const int zero = 0;
     if (warp == 0) {
       mbar_wait(&bars.q_full, 0, &zero, tmo);
-      for (int i = (k_issued > C::kStages ? k_issued - C::kStages : 0); i < k_issued; ++i)
-        mbar_wait(&bars.k_full[i % C::kStages], (uint32_t)(i / C::kStages) & 1u, &zero, tmo);
-      for (int i = (v_issued > C::kStages ? v_issued - C::kStages : 0); i < v_issued; ++i) {
+      for (int i = (k_issued > C::kKStages ? k_issued - C::kKStages : 0); i < k_issued; ++i)
+        mbar_wait(&bars.k_full[i % C::kKStages], (uint32_t)(i / C::kKStages) & 1u, &zero, tmo);
+      for (int i = (v_issued > C::kVStages ? v_issued - C::kVStages : 0); i < v_issued; ++i) {
         if (p.fault_mode == 1 && i == 1) continue;  // the copy the test hook withheld
-        mbar_wait(&bars.v_full[i % C::kStages], (uint32_t)(i / C::kStages) & 1u, &zero, tmo);
+        mbar_wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u, &zero, tmo);
       }
     } else if (warp == 1) {
       mma_commit(&bars.drain);

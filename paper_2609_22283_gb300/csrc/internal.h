@@ -37,6 +37,7 @@ struct alignas(128) AttnParams {
   int32_t Tpad;         // T rounded up to kTile: rows per (slot, K|V, head)
   int32_t H;
   int32_t n_qt;         // query tiles per node = ceil(T / kTile)
+  int32_t n_qp;         // work units per (node, head): query-tile pairs = ceil(n_qt / 2)
   int32_t n_nodes;
   int32_t nt_slot;      // key tiles per slot = Tpad / kTile
   int32_t valid_last;   // valid key rows in the last tile of a slot

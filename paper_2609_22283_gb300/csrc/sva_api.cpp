@@ -559,13 +559,14 @@ sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes
   p.Tpad = c->L.Tpad;
   p.H = g.num_heads;
   p.n_qt = (c->L.T + sva::kTile - 1) / sva::kTile;
+  p.n_qp = (p.n_qt + 1) / 2;
   p.n_nodes = n_nodes;
   p.nt_slot = c->L.Tpad / sva::kTile;
   p.valid_last = c->L.T - (p.nt_slot - 1) * sva::kTile;
   p.fault_mode = c->fault_mode;
   p.timeout_ns = c->timeout_ns;
   c->fault_mode = 0;
-  const long long grid = (long long)g.num_heads * n_nodes * p.n_qt;
+  const long long grid = (long long)g.num_heads * n_nodes * p.n_qp;
   cudaError_t e = sva::launch_attend(p, g.head_dim, (int)grid, reinterpret_cast<cudaStream_t>(s));
   if (e != cudaSuccess) return cuda_fail(e, "attend launch");
   return ok();
