@@ -189,6 +189,23 @@ sva_status sva_rope_kv_write(sva_cache* c, const sva_node* nodes, int32_t n_node
 sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* q,
                             void* out, float* lse, float scale, sva_stream s);
 
+/* Bytes of the optional split workspace of a cache (0 if c is NULL).  With
+ * a workspace attached, sva_attend_nodes may divide each (node, head,
+ * query-tile pair) work unit into up to 4 contiguous key ranges computed by
+ * separate CTAs and merged on the device (the softmax of Eq. 4 recombined
+ * from per-range maxima and sums), which fills the GPU when a launch has
+ * too few work units; results agree with the unsplit computation to
+ * rounding. */
+size_t sva_attend_workspace_bytes(const sva_cache* c);
+
+/* Attaches a caller-owned device buffer of at least
+ * sva_attend_workspace_bytes(c) bytes (256-byte aligned, on the cache's
+ * device) as the split workspace, or detaches it when dev_buf is NULL.
+ * Zeroes the buffer's counters (synchronous).  The buffer must outlive its
+ * use; launches on one cache that overlap on the GPU must not share it.
+ * Errors: INVALID_ARGUMENT, CUDA. */
+sva_status sva_cache_set_workspace(sva_cache* c, void* dev_buf, size_t bytes);
+
 /* Synchronizes `s`, then reads and clears the device status word: returns
  * DEVICE_TIMEOUT if a kernel gave up a bounded wait since the last poll,
  * CUDA if the stream reported an error, else OK. */

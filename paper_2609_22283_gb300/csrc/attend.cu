@@ -24,6 +24,11 @@
 // hide behind.  A commit that completes S_b of tile i also implies PV_b of
 // tile i-1 is complete (MMAs execute in issue order), so the rescale of O_b
 // needs no extra barrier.
+// A unit may be split into n_split contiguous key ranges (when there are too
+// few units to fill the GPU's waves): each split CTA writes its normalised
+// partial O with its row max and sum to the workspace and bumps the unit's
+// arrival counter; the last to arrive merges the partials (the usual
+// log-sum-exp combination) and writes the output, then resets the counter.
 // All waits are bounded (1 s by default): on expiry the CTA records
 // SVA_ERR_DEVICE_TIMEOUT in the status word, drains its own copies and MMAs,
 // frees TMEM and exits.
@@ -128,18 +133,23 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
   __shared__ Bars bars;
   __shared__ uint32_t tmem_base_sh;
   __shared__ volatile int abort_flag;
+  __shared__ int last_split;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
-  // Work unit, head-major so the CTAs that share a head's K/V run together.
-  const int unit = blockIdx.x;
+  // Work unit, head-major so the CTAs that share a head's K/V run together;
+  // the splits of a unit are adjacent.
+  const int split = blockIdx.x % p.n_split;
+  const int unit = blockIdx.x / p.n_split;
   const int qp = unit % p.n_qp;
   const int rest = unit / p.n_qp;
   const int ni = rest % p.n_nodes;
   const int h = rest / p.n_nodes;
   const AttnNode& nd = p.nodes[ni];
-  const int n_tiles = nd.n_kv * p.nt_slot;
+  const int n_all = nd.n_kv * p.nt_slot;  // key tiles of the node
+  const int t_begin = (int)((long long)split * n_all / p.n_split);
+  const int n_tiles = (int)((long long)(split + 1) * n_all / p.n_split) - t_begin;
   const int qt0 = 2 * qp;
   const bool has_q1 = qt0 + 1 < p.n_qt;
 
@@ -193,14 +203,15 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
                       (qt0 + 1) * kTile, nd.q_index);
       }
       const uint64_t keep = l2_policy_evict_last();
-      for (int i = 0; i < n_tiles; ++i) {
-        const int ks = i % C::kKStages;
-        const int vs = i % C::kVStages;
+      for (int j = 0; j < n_tiles; ++j) {
+        const int i = t_begin + j;  // key tile of the node
+        const int ks = j % C::kKStages;
+        const int vs = j % C::kVStages;
         const int slot = nd.slot[i / p.nt_slot];
         const int t = i - (i / p.nt_slot) * p.nt_slot;
         const int row_k = ((slot * 2 + 0) * p.H + h) * p.Tpad + t * kTile;
         const int row_v = row_k + p.H * p.Tpad;
-        if (!mbar_wait(&bars.k_empty[ks], ((uint32_t)(i / C::kKStages) & 1u) ^ 1u, &abort_flag,
+        if (!mbar_wait(&bars.k_empty[ks], ((uint32_t)(j / C::kKStages) & 1u) ^ 1u, &abort_flag,
                        tmo)) {
           record_timeout(p, &abort_flag);
           break;
@@ -210,22 +221,22 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         for (int b = 0; b < C::kBoxes; ++b)
           tma_load_2d_hint(sK + ks * C::kTileBytes + b * C::kBoxBytes, &p.tmap_kv,
                            &bars.k_full[ks], b * 64, row_k, keep);
-        k_issued = i + 1;
-        if (!mbar_wait(&bars.v_empty[vs], ((uint32_t)(i / C::kVStages) & 1u) ^ 1u, &abort_flag,
+        k_issued = j + 1;
+        if (!mbar_wait(&bars.v_empty[vs], ((uint32_t)(j / C::kVStages) & 1u) ^ 1u, &abort_flag,
                        tmo)) {
           record_timeout(p, &abort_flag);
           break;
         }
-        // fault_mode 1 (test hook): withhold the V copy of tile 1, so the
-        // MMA issuer's bounded wait on it expires.
-        if (!(p.fault_mode == 1 && i == 1)) {
+        // fault_mode 1 (test hook): withhold the V copy of the second tile,
+        // so the MMA issuer's bounded wait on it expires.
+        if (!(p.fault_mode == 1 && j == 1)) {
           mbar_arrive_expect_tx(&bars.v_full[vs], C::kTileBytes);
 #pragma unroll
           for (int b = 0; b < C::kBoxes; ++b)
             tma_load_2d_hint(sV + vs * C::kTileBytes + b * C::kBoxBytes, &p.tmap_kv,
                              &bars.v_full[vs], b * 64, row_v, keep);
         }
-        v_issued = i + 1;
+        v_issued = j + 1;
       }
     }
   } else if (warp == 1) {
@@ -327,7 +338,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         ok = __all_sync(0xffffffffu, ok);
         if (!ok) break;
         tc_fence_after();
-        const int t = i % p.nt_slot;
+        const int t = (t_begin + i) % p.nt_slot;  // key tile inside its slot
         const int valid = (t == p.nt_slot - 1) ? p.valid_last : kTile;
         float m_tile;
         {
@@ -427,36 +438,114 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         ok = mbar_wait(&bars.o_final, 0, &abort_flag, tmo);
         ok = __all_sync(0xffffffffu, ok);
       }
-      if (!ok) {
-        record_timeout(p, &abort_flag);
-      } else {
-        tc_fence_after();
-        const int token = (qt0 + b) * kTile + row;
-        const bool in_range = token < p.T;
-        const float inv_l = 1.0f / l;
-        __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(p.out) +
-                              (((size_t)nd.q_index * p.T + token) * p.H + h) * D;
+      if (!ok) record_timeout(p, &abort_flag);
+      const int token = (qt0 + b) * kTile + row;
+      const bool in_range = token < p.T;
+      __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(p.out) +
+                            (((size_t)nd.q_index * p.T + token) * p.H + h) * D;
+      float* lse_at = p.lse ? p.lse + ((size_t)nd.q_index * p.H + h) * p.T + token : nullptr;
+      if (p.n_split == 1) {
+        if (ok) {
+          tc_fence_after();
+          const float inv_l = 1.0f / l;
 #pragma unroll
-        for (int c = 0; c < D / 32; ++c) {
-          uint32_t o[32];
-          tmem_ld32(ocol + c * 32, o);
-          tmem_wait_ld(o);
-          if (in_range) {
-            uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t o[32];
+            tmem_ld32(ocol + c * 32, o);
+            tmem_wait_ld(o);
+            if (in_range) {
+              uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
 #pragma unroll
-            for (int v = 0; v < 4; ++v) {
-              uint4 w;
-              w.x = pack_bf16(__uint_as_float(o[v * 8 + 0]) * inv_l, __uint_as_float(o[v * 8 + 1]) * inv_l);
-              w.y = pack_bf16(__uint_as_float(o[v * 8 + 2]) * inv_l, __uint_as_float(o[v * 8 + 3]) * inv_l);
-              w.z = pack_bf16(__uint_as_float(o[v * 8 + 4]) * inv_l, __uint_as_float(o[v * 8 + 5]) * inv_l);
-              w.w = pack_bf16(__uint_as_float(o[v * 8 + 6]) * inv_l, __uint_as_float(o[v * 8 + 7]) * inv_l);
-              dst[v] = w;
+              for (int v = 0; v < 4; ++v) {
+                uint4 w;
+                w.x = pack_bf16(__uint_as_float(o[v * 8 + 0]) * inv_l, __uint_as_float(o[v * 8 + 1]) * inv_l);
+                w.y = pack_bf16(__uint_as_float(o[v * 8 + 2]) * inv_l, __uint_as_float(o[v * 8 + 3]) * inv_l);
+                w.z = pack_bf16(__uint_as_float(o[v * 8 + 4]) * inv_l, __uint_as_float(o[v * 8 + 5]) * inv_l);
+                w.w = pack_bf16(__uint_as_float(o[v * 8 + 6]) * inv_l, __uint_as_float(o[v * 8 + 7]) * inv_l);
+                dst[v] = w;
+              }
             }
           }
+          if (lse_at != nullptr && in_range) *lse_at = (m + __log2f(l)) * 0.69314718055994531f;
         }
-        if (p.lse != nullptr && in_range) {
-          p.lse[((size_t)nd.q_index * p.H + h) * p.T + token] =
-              (m + __log2f(l)) * 0.69314718055994531f;
+      } else {
+        // Split unit.  Partial layout per (unit, split): O as [D/4][256]
+        // float4 (rows of both query tiles), then m[256], then l[256].
+        constexpr size_t kItem = (size_t)256 * (D + 2);
+        const int r = b * 128 + row;
+        float* part = p.ws + ((size_t)unit * p.n_split + split) * kItem;
+        if (ok) {
+          tc_fence_after();
+          const float inv_l = 1.0f / l;
+          float4* part4 = reinterpret_cast<float4*>(part);
+#pragma unroll
+          for (int c = 0; c < D / 32; ++c) {
+            uint32_t o[32];
+            tmem_ld32(ocol + c * 32, o);
+            tmem_wait_ld(o);
+#pragma unroll
+            for (int v = 0; v < 8; ++v)
+              part4[(c * 8 + v) * 256 + r] =
+                  make_float4(__uint_as_float(o[v * 4 + 0]) * inv_l, __uint_as_float(o[v * 4 + 1]) * inv_l,
+                              __uint_as_float(o[v * 4 + 2]) * inv_l, __uint_as_float(o[v * 4 + 3]) * inv_l);
+          }
+          part[D * 256 + r] = m;
+          part[D * 256 + 256 + r] = l;
+        }
+        __threadfence();
+        // Every softmax thread of the CTA passes both barriers, whatever its
+        // wait results were, so none can be left waiting here.
+        const uint32_t nsoft = has_q1 ? 256u : 128u;
+        asm volatile("bar.sync 1, %0;" ::"r"(nsoft) : "memory");
+        if (threadIdx.x == 64) {
+          int last = 0;
+          if (!abort_flag) last = atomicAdd(&p.ws_count[unit], 1) == p.n_split - 1;
+          last_split = last;
+        }
+        asm volatile("bar.sync 1, %0;" ::"r"(nsoft) : "memory");
+        if (last_split) {
+          __threadfence();
+          const float* base = p.ws + (size_t)unit * p.n_split * kItem;
+          float mk[kMaxSplit], wk[kMaxSplit];
+          float M = -INFINITY;
+#pragma unroll
+          for (int k = 0; k < kMaxSplit; ++k) {
+            mk[k] = k < p.n_split ? __ldcg(base + k * kItem + D * 256 + r) : -INFINITY;
+            M = fmaxf(M, mk[k]);
+          }
+          float L = 0.0f;
+#pragma unroll
+          for (int k = 0; k < kMaxSplit; ++k) {
+            wk[k] = k < p.n_split ? __ldcg(base + k * kItem + D * 256 + 256 + r) * ex2(mk[k] - M)
+                                  : 0.0f;
+            L += wk[k];
+          }
+          const float inv_L = 1.0f / L;
+#pragma unroll
+          for (int k = 0; k < kMaxSplit; ++k) wk[k] *= inv_L;
+          if (in_range) {
+#pragma unroll 4
+            for (int c8 = 0; c8 < D / 8; ++c8) {
+              float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+              for (int k = 0; k < kMaxSplit; ++k) {
+                if (k >= p.n_split) break;
+                const float4* b4 = reinterpret_cast<const float4*>(base + k * kItem);
+                const float4 x = __ldcg(b4 + (c8 * 2 + 0) * 256 + r);
+                const float4 y = __ldcg(b4 + (c8 * 2 + 1) * 256 + r);
+                a[0] += wk[k] * x.x; a[1] += wk[k] * x.y; a[2] += wk[k] * x.z; a[3] += wk[k] * x.w;
+                a[4] += wk[k] * y.x; a[5] += wk[k] * y.y; a[6] += wk[k] * y.z; a[7] += wk[k] * y.w;
+              }
+              uint4 w;
+              w.x = pack_bf16(a[0], a[1]);
+              w.y = pack_bf16(a[2], a[3]);
+              w.z = pack_bf16(a[4], a[5]);
+              w.w = pack_bf16(a[6], a[7]);
+              reinterpret_cast<uint4*>(orow)[c8] = w;
+            }
+            if (lse_at != nullptr) *lse_at = (M + __log2f(L)) * 0.69314718055994531f;
+          }
+          if (threadIdx.x == 64) p.ws_count[unit] = 0;  // ready for the next launch
         }
       }
     }

@@ -12,6 +12,7 @@
 namespace sva {
 
 constexpr int kTile = 128;  // query rows per Q tile and key rows per K/V tile
+constexpr int kMaxSplit = 4;  // key-range splits of one work unit
 constexpr uint64_t kDefaultWaitTimeoutNs = 1000000000ull;  // bounded device waits: 1 s
 
 // Device status word values (a subset of sva_status).
@@ -42,6 +43,9 @@ struct alignas(128) AttnParams {
   int32_t nt_slot;      // key tiles per slot = Tpad / kTile
   int32_t valid_last;   // valid key rows in the last tile of a slot
   int32_t fault_mode;   // 0 in production; see sva_api.cpp
+  int32_t n_split;      // key-range splits per work unit (1 = no split)
+  float* ws;            // split partials [unit][split][(d + 2) * 256] fp32, or null
+  int* ws_count;        // per-unit arrival counters, zero between launches, or null
   uint64_t timeout_ns;
   AttnNode nodes[SVA_MAX_NODES];
 };

@@ -5,6 +5,7 @@
 // and availability (Eq. 7), the validation of every launch, the TMA
 // descriptors, and the launches of the two kernels.  Device memory is always
 // the caller's.
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -208,6 +209,7 @@ struct sva_cache {
   CUtensorMap tmap_q{};
   int fault_mode = 0;  // one-shot test hook, see sva_debug_inject
   uint64_t timeout_ns = sva::kDefaultWaitTimeoutNs;
+  char* ws = nullptr;  // caller's split workspace (sva_cache_set_workspace), or null
 };
 
 namespace {
@@ -234,6 +236,36 @@ sva_status check_own(const sva_cache* c, const sva_node& n, int i, bool need_res
   if (need_resident && !s.resident)
     return fail(SVA_ERR_NOT_RESIDENT, "node %d: own_slot %d has not been written", i, n.own_slot);
   return SVA_OK;
+}
+
+// Split workspace: room for 4 waves of split work items (one per SM and
+// wave), each 256 query rows x (d + 2) fp32, after one arrival counter per
+// item.
+int ws_items(const sva_cache* c) { return 4 * c->num_sms; }
+size_t ws_item_bytes(const sva_cache* c) { return (size_t)256 * (c->g.head_dim + 2) * 4; }
+size_t ws_counter_bytes(const sva_cache* c) { return round_up((size_t)ws_items(c) * 4, 256); }
+size_t ws_total_bytes(const sva_cache* c) {
+  return ws_counter_bytes(c) + (size_t)ws_items(c) * ws_item_bytes(c);
+}
+
+// Splits per work unit: the smallest s in 1..kMaxSplit minimising the wave
+// count per split, ceil(units * s / SMs) / s, subject to the workspace
+// capacity and to at least 4 key tiles per split.
+int choose_split(const sva_cache* c, long long units, int min_tiles) {
+  if (c->ws == nullptr) return 1;
+  const long long sms = c->num_sms;
+  double best = (double)((units + sms - 1) / sms);
+  int best_s = 1;
+  for (int s = 2; s <= sva::kMaxSplit; ++s) {
+    const long long items = units * s;
+    if (items > ws_items(c) || min_tiles / s < 4) break;
+    const double cost = (double)((items + sms - 1) / sms) / s;
+    if (cost < best - 1e-9) {
+      best = cost;
+      best_s = s;
+    }
+  }
+  return best_s;
 }
 
 }  // namespace
@@ -566,7 +598,15 @@ sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes
   p.fault_mode = c->fault_mode;
   p.timeout_ns = c->timeout_ns;
   c->fault_mode = 0;
-  const long long grid = (long long)g.num_heads * n_nodes * p.n_qp;
+  int min_tiles = 1 << 30;
+  for (int i = 0; i < n_nodes; ++i) min_tiles = std::min(min_tiles, p.nodes[i].n_kv * p.nt_slot);
+  const long long units = (long long)g.num_heads * n_nodes * p.n_qp;
+  p.n_split = choose_split(c, units, min_tiles);
+  if (p.n_split > 1) {
+    p.ws_count = reinterpret_cast<int*>(c->ws);
+    p.ws = reinterpret_cast<float*>(c->ws + ws_counter_bytes(c));
+  }
+  const long long grid = units * p.n_split;
   cudaError_t e = sva::launch_attend(p, g.head_dim, (int)grid, reinterpret_cast<cudaStream_t>(s));
   if (e != cudaSuccess) return cuda_fail(e, "attend launch");
   return ok();
@@ -585,10 +625,45 @@ sva_status sva_poll_device_status(sva_cache* c, sva_stream s) {
     e = cudaMemset(c->base + c->L.status, 0, sizeof(int));
     if (e == cudaSuccess) e = cudaDeviceSynchronize();
     if (e != cudaSuccess) return cuda_fail(e, "clearing the status word");
+    if (c->ws != nullptr) {
+      // a timed-out split unit may have left its arrival counter non-zero
+      e = cudaMemset(c->ws, 0, ws_counter_bytes(c));
+      if (e == cudaSuccess) e = cudaDeviceSynchronize();
+      if (e != cudaSuccess) return cuda_fail(e, "clearing the split counters");
+    }
     if (word == SVA_ERR_DEVICE_TIMEOUT)
       return fail(SVA_ERR_DEVICE_TIMEOUT, "a kernel gave up a bounded wait; its outputs are invalid");
     return fail(SVA_ERR_CUDA, "device status word %d", word);
   }
+  return ok();
+}
+
+size_t sva_attend_workspace_bytes(const sva_cache* c) {
+  if (c == nullptr) return 0;
+  return ws_total_bytes(c);
+}
+
+sva_status sva_cache_set_workspace(sva_cache* c, void* dev_buf, size_t bytes) {
+  if (c == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "NULL cache");
+  if (dev_buf == nullptr) {
+    c->ws = nullptr;
+    return ok();
+  }
+  if ((reinterpret_cast<uintptr_t>(dev_buf) & 255u) != 0)
+    return fail(SVA_ERR_INVALID_ARGUMENT, "workspace must be 256-byte aligned");
+  if (bytes < ws_total_bytes(c))
+    return fail(SVA_ERR_INVALID_ARGUMENT, "workspace of %zu bytes is smaller than the %zu needed",
+                bytes, ws_total_bytes(c));
+  cudaPointerAttributes attr;
+  cudaError_t e = cudaPointerGetAttributes(&attr, dev_buf);
+  if (e != cudaSuccess || attr.type != cudaMemoryTypeDevice || attr.device != c->device) {
+    cudaGetLastError();
+    return fail(SVA_ERR_INVALID_ARGUMENT, "workspace is not device memory of the cache's device");
+  }
+  e = cudaMemset(dev_buf, 0, ws_counter_bytes(c));
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(e, "zeroing the workspace counters");
+  c->ws = static_cast<char*>(dev_buf);
   return ok();
 }
 

@@ -28,11 +28,15 @@ def geometry_for(w: Workload, spare_slots: int = 2) -> sva.sva_geometry:
 
 
 class Step:
-    def __init__(self, w: Workload, device: str = "cuda", spare_slots: int = 2):
+    def __init__(self, w: Workload, device: str = "cuda", spare_slots: int = 2,
+                 workspace: bool = True):
         self.w = w
         self.device = torch.device(device)
         self.policy = sva.POLICIES[w.policy]
         self.cache = sva.Cache(geometry_for(w, spare_slots), device=self.device)
+        if workspace:
+            ws = torch.empty(self.cache.workspace_bytes(), dtype=torch.uint8, device=self.device)
+            self.cache.set_workspace(ws)
         self.own = {}
         self.scale = 1.0 / math.sqrt(w.d)
 

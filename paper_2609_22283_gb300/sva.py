@@ -35,7 +35,8 @@ MAX_NODES = 64
 
 EXPORTED = ("sva_cache_bytes", "sva_cache_create", "sva_cache_bind", "sva_cache_lookup",
             "sva_cache_release", "sva_select_context", "sva_pipeline_round", "sva_check_pipeline",
-            "sva_rope_kv_write", "sva_attend_nodes", "sva_poll_device_status", "sva_debug_inject",
+            "sva_rope_kv_write", "sva_attend_nodes", "sva_attend_workspace_bytes",
+            "sva_cache_set_workspace", "sva_poll_device_status", "sva_debug_inject",
             "sva_destroy", "sva_last_error")
 
 
@@ -84,6 +85,8 @@ def load(path: str = LIB_PATH):
         "sva_check_pipeline": ([i32, i32, i32, i32, pi32, pi32], i32),
         "sva_rope_kv_write": ([p, pn, i32, p, p, p, p], i32),
         "sva_attend_nodes": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
+        "sva_attend_workspace_bytes": ([p], ctypes.c_size_t),
+        "sva_cache_set_workspace": ([p, p, ctypes.c_size_t], i32),
         "sva_poll_device_status": ([p, p], i32),
         "sva_debug_inject": ([p, i32, ctypes.c_double], i32),
         "sva_destroy": ([p], i32),
@@ -256,6 +259,19 @@ class Cache:
                                    ctypes.c_void_p(lse.data_ptr() if lse is not None else 0),
                                    float(scale), ctypes.c_void_p(_stream_handle(stream)))
         _check(st)
+
+    def workspace_bytes(self) -> int:
+        return int(_lib.sva_attend_workspace_bytes(self.handle))
+
+    def set_workspace(self, buf: torch.Tensor | None):
+        """Attaches a caller-owned split workspace (a CUDA uint8 tensor), or detaches it."""
+        if buf is None:
+            _check(_lib.sva_cache_set_workspace(self.handle, None, 0))
+            self.ws = None
+            return
+        nbytes = buf.numel() * buf.element_size()
+        _check(_lib.sva_cache_set_workspace(self.handle, ctypes.c_void_p(buf.data_ptr()), nbytes))
+        self.ws = buf
 
     def poll(self, stream=None) -> int:
         """sva_poll_device_status: returns the status code (0 = OK)."""
