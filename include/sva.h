@@ -206,6 +206,32 @@ size_t sva_attend_workspace_bytes(const sva_cache* c);
  * Errors: INVALID_ARGUMENT, CUDA. */
 sva_status sva_cache_set_workspace(sva_cache* c, void* dev_buf, size_t bytes);
 
+/* sva_attend_nodes for callers that may not allocate device memory at all:
+ * for example a plugin that its host framework hands only input and output
+ * buffers, with every other byte of device memory budgeted by that
+ * framework, or a serving loop that forbids cudaMalloc because it can block
+ * and synchronise the device.  Such a caller cannot provide the split
+ * workspace of sva_cache_set_workspace.  This entry point takes the same
+ * arguments and gives the same results (within rounding) as
+ * sva_attend_nodes with a workspace attached, but keeps its key-range
+ * partials and arrival counters in a scratch array that the library
+ * declares in device memory itself (32 MiB, held by every GPU that loads
+ * the library until the process exits).  It allocates nothing and calls no
+ * allocating routine.  Launches whose split plan needs more than 32 MiB of
+ * scratch are rejected with SVA_ERR_CAPACITY and launch nothing; launches
+ * that need no split use no scratch and are never rejected for size.
+ * Each call clears the array's counters on `s` before its kernel; the
+ * partials left by one call are overwritten by the next.  All calls on a
+ * device share the one array, so calls whose kernels can overlap on the
+ * GPU (different streams without ordering between them) race and must not
+ * be issued.  The first call on a device looks up the array's device
+ * address (cudaGetSymbolAddress); make that first call before any stream
+ * capture.  The paper has no counterpart of this entry point.
+ * Errors: as sva_attend_nodes, plus CAPACITY for a plan that does not fit. */
+sva_status sva_attend_nodes_noalloc(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
+                                    const void* q, void* out, float* lse, float scale,
+                                    sva_stream s);
+
 /* Synchronizes `s`, then reads and clears the device status word: returns
  * DEVICE_TIMEOUT if a kernel gave up a bounded wait since the last poll,
  * CUDA if the stream reported an error, else OK. */

@@ -69,6 +69,13 @@ struct RopeParams {
   RopeNode nodes[SVA_MAX_NODES];
 };
 
+// Size of the library-owned split scratch used by sva_attend_nodes_noalloc.
+constexpr size_t kStaticScratchBytes = (size_t)32 << 20;
+
+// Device address of that scratch on `device` (the current device); the
+// first call on a device looks it up.  Defined in attend_noalloc.cu.
+cudaError_t static_split_scratch(int device, void** ptr);
+
 // Launchers (defined in the .cu files).  They return the launch error.
 cudaError_t launch_attend(const AttnParams& p, int head_dim, int grid, cudaStream_t s);
 cudaError_t launch_rope_kv(const RopeParams& p, cudaStream_t s);

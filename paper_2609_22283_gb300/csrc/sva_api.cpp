@@ -612,6 +612,130 @@ sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes
   return ok();
 }
 
+// Attention with the split scratch taken from the library's own device
+// array instead of a caller-attached workspace (see include/sva.h).  The
+// checks and the launch parameters are those of sva_attend_nodes.
+sva_status sva_attend_nodes_noalloc(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
+                                    const void* q, void* out, float* lse, float scale,
+                                    sva_stream s) {
+  if (c == nullptr || nodes == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "NULL argument");
+  if (n_nodes < 1) return fail(SVA_ERR_INVALID_ARGUMENT, "n_nodes %d < 1", n_nodes);
+  if (n_nodes > SVA_MAX_NODES)
+    return fail(SVA_ERR_CAPACITY, "n_nodes %d > SVA_MAX_NODES (%d)", n_nodes, SVA_MAX_NODES);
+  if (q == nullptr || out == nullptr || !aligned16(q) || !aligned16(out) ||
+      (lse != nullptr && (reinterpret_cast<uintptr_t>(lse) & 3u) != 0))
+    return fail(SVA_ERR_INVALID_ARGUMENT, "q/out must be non-NULL and 16-byte aligned, lse 4-byte aligned");
+  if (!std::isfinite(scale) || !(scale > 0.0f))
+    return fail(SVA_ERR_INVALID_ARGUMENT, "scale must be finite and > 0");
+  sva_status st = check_device(c);
+  if (st != SVA_OK) return st;
+  const sva_geometry& g = c->g;
+
+  static thread_local sva::AttnParams p;
+  std::memset(&p, 0, sizeof(p));
+  for (int i = 0; i < n_nodes; ++i) {
+    const sva_node& n = nodes[i];
+    st = check_own(c, n, i, true);
+    if (st != SVA_OK) return st;
+    if (n.n_ctx < 0 || n.n_ctx > SVA_MAX_CTX)
+      return fail(SVA_ERR_CAPACITY, "node %d: n_ctx %d outside 0..%d", i, n.n_ctx, SVA_MAX_CTX);
+    sva::AttnNode& a = p.nodes[i];
+    a.q_index = i;
+    a.slot[0] = n.own_slot;
+    int nkv = 1;
+    for (int k = 0; k < n.n_ctx; ++k) {
+      const int32_t cs = n.ctx_slot[k];
+      if (cs < 0 || cs >= g.num_slots)
+        return fail(SVA_ERR_INVALID_ARGUMENT, "node %d ctx %d: slot %d out of range", i, k, cs);
+      const SlotInfo& si = c->slots[cs];
+      if (!si.bound || !si.resident)
+        return fail(SVA_ERR_NOT_RESIDENT, "node %d ctx %d: slot %d is %s", i, k, cs,
+                    si.bound ? "bound but not written" : "not bound");
+      if (si.seq != n.seq || si.chunk >= n.chunk)
+        return fail(SVA_ERR_CAUSALITY,
+                    "node %d (seq %d, chunk %d) ctx %d: slot %d holds (seq %d, chunk %d), not a "
+                    "past chunk of the same sequence",
+                    i, n.seq, n.chunk, k, cs, si.seq, si.chunk);
+      if (cs == n.own_slot)
+        return fail(SVA_ERR_INVALID_ARGUMENT, "node %d ctx %d repeats the own slot", i, k);
+      for (int k2 = 0; k2 < k; ++k2)
+        if (n.ctx_slot[k2] == cs)
+          return fail(SVA_ERR_INVALID_ARGUMENT, "node %d: slot %d listed twice", i, cs);
+      if (n.ctx_visible[k]) a.slot[nkv++] = cs;
+    }
+    a.n_kv = nkv;
+  }
+  p.n_qt = (c->L.T + sva::kTile - 1) / sva::kTile;
+  p.n_qp = (p.n_qt + 1) / 2;
+  p.nt_slot = c->L.Tpad / sva::kTile;
+  int min_tiles = 1 << 30;
+  for (int i = 0; i < n_nodes; ++i) min_tiles = std::min(min_tiles, p.nodes[i].n_kv * p.nt_slot);
+  const long long units = (long long)g.num_heads * n_nodes * p.n_qp;
+
+  // The split plan a full workspace would get; its scratch must fit the array.
+  const long long sms = c->num_sms;
+  double best = (double)((units + sms - 1) / sms);
+  int n_split = 1;
+  for (int sp = 2; sp <= sva::kMaxSplit; ++sp) {
+    const long long items = units * sp;
+    if (items > ws_items(c) || min_tiles / sp < 4) break;
+    const double cost = (double)((items + sms - 1) / sms) / sp;
+    if (cost < best - 1e-9) {
+      best = cost;
+      n_split = sp;
+    }
+  }
+  void* scratch = nullptr;
+  size_t counter_bytes = 0;
+  if (n_split > 1) {
+    counter_bytes = round_up((size_t)units * 4, 256);
+    const size_t need = counter_bytes + (size_t)units * n_split * ws_item_bytes(c);
+    if (need > sva::kStaticScratchBytes)
+      return fail(SVA_ERR_CAPACITY,
+                  "this launch splits %lld work units %d ways and needs %zu bytes of scratch; the "
+                  "library's static scratch holds %zu bytes (use sva_attend_nodes with a "
+                  "workspace for launches this large)",
+                  units, n_split, need, sva::kStaticScratchBytes);
+    cudaError_t e = sva::static_split_scratch(c->device, &scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(split scratch)");
+    // the arrival counters must start at zero; the array keeps whatever the
+    // previous call left in it
+    e = cudaMemsetAsync(scratch, 0, counter_bytes, reinterpret_cast<cudaStream_t>(s));
+    if (e != cudaSuccess) return cuda_fail(e, "clearing the split counters");
+  }
+  if (c->q_cached != q || c->q_cached_n != n_nodes) {
+    st = encode_4d_q(&c->tmap_q, q, g, c->L.T, n_nodes);
+    if (st != SVA_OK) {
+      c->q_cached = nullptr;
+      return st;
+    }
+    c->q_cached = q;
+    c->q_cached_n = n_nodes;
+  }
+  p.tmap_q = c->tmap_q;
+  p.tmap_kv = c->tmap_kv;
+  p.out = out;
+  p.lse = lse;
+  p.status = reinterpret_cast<int*>(c->base + c->L.status);
+  p.scale_log2 = scale * 1.4426950408889634f;
+  p.T = c->L.T;
+  p.Tpad = c->L.Tpad;
+  p.H = g.num_heads;
+  p.n_nodes = n_nodes;
+  p.valid_last = c->L.T - (p.nt_slot - 1) * sva::kTile;
+  p.fault_mode = 0;
+  p.timeout_ns = c->timeout_ns;
+  p.n_split = n_split;
+  if (n_split > 1) {
+    p.ws_count = static_cast<int*>(scratch);
+    p.ws = reinterpret_cast<float*>(static_cast<char*>(scratch) + counter_bytes);
+  }
+  const long long grid = units * n_split;
+  cudaError_t e = sva::launch_attend(p, g.head_dim, (int)grid, reinterpret_cast<cudaStream_t>(s));
+  if (e != cudaSuccess) return cuda_fail(e, "attend launch");
+  return ok();
+}
+
 sva_status sva_poll_device_status(sva_cache* c, sva_stream s) {
   if (c == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "NULL argument");
   sva_status st = check_device(c);

@@ -36,8 +36,8 @@ MAX_NODES = 64
 EXPORTED = ("sva_cache_bytes", "sva_cache_create", "sva_cache_bind", "sva_cache_lookup",
             "sva_cache_release", "sva_select_context", "sva_pipeline_round", "sva_check_pipeline",
             "sva_rope_kv_write", "sva_attend_nodes", "sva_attend_workspace_bytes",
-            "sva_cache_set_workspace", "sva_poll_device_status", "sva_debug_inject",
-            "sva_destroy", "sva_last_error")
+            "sva_cache_set_workspace", "sva_attend_nodes_noalloc", "sva_poll_device_status",
+            "sva_debug_inject", "sva_destroy", "sva_last_error")
 
 
 class SvaError(RuntimeError):
@@ -86,6 +86,7 @@ def load(path: str = LIB_PATH):
         "sva_rope_kv_write": ([p, pn, i32, p, p, p, p], i32),
         "sva_attend_nodes": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
         "sva_attend_workspace_bytes": ([p], ctypes.c_size_t),
+        "sva_attend_nodes_noalloc": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
         "sva_cache_set_workspace": ([p, p, ctypes.c_size_t], i32),
         "sva_poll_device_status": ([p, p], i32),
         "sva_debug_inject": ([p, i32, ctypes.c_double], i32),
