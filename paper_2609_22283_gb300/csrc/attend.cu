@@ -14,7 +14,7 @@
 //   warp 0     TMA producer: Q0/Q1 once, then K and V tiles of the slot list
 //              into rings of shared-memory stages (128B swizzle);
 //   warp 1     MMA issuer (one thread) and TMEM owner;
-//   warps 2-5  softmax of Q0, warps 6-9 softmax of Q1: one query row per
+//   warps 4-7  softmax of Q0, warps 8-11 softmax of Q1: one query row per
 //              thread; S from TMEM, fp32 online softmax in the log2 domain
 //              with a lazy rescale of O, P written back over S as bf16; then
 //              the epilogue (O / l to bf16 global, optional LSE).
@@ -63,8 +63,29 @@ struct AttnCfg {
 __device__ __forceinline__ uint32_t col_s(int b) { return b ? 128u : 0u; }
 __device__ __forceinline__ uint32_t col_o(int b) { return b ? 384u : 256u; }
 
-constexpr int kThreads = 320;
+// 12 warps: warpgroup 0 = TMA producer (warp 0), MMA issuer (warp 1), two
+// idle warps; warpgroups 1 and 2 = softmax of query tiles 0 and 1.  The
+// launch gives every thread kLaunchRegs registers; warpgroup 0 then gives
+// registers back (setmaxnreg.dec to kRegsLow) and the softmax warpgroups
+// take them (setmaxnreg.inc to kRegsHigh), so a softmax thread can hold a
+// whole 128-key row of S.  The split must fit the launch's pool:
+// 4*32*kRegsLow + 8*32*kRegsHigh <= 384*kLaunchRegs, checked at launch.
+constexpr int kThreads = 384;
+constexpr int kLaunchRegs = 168;
+constexpr int kRegsLow = 72;
+constexpr int kRegsHigh = 216;
+static_assert(4 * 32 * kRegsLow + 8 * 32 * kRegsHigh <= kThreads * kLaunchRegs, "register split");
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: P <= 2^8 between rescales
+
+template <int N>
+__device__ __forceinline__ void regs_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(N));
+}
+
+template <int N>
+__device__ __forceinline__ void regs_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(N));
+}
 
 __device__ __forceinline__ float ex2(float x) {
   float y;
@@ -188,7 +209,9 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
   uint8_t* sV = smem + C::kOffV;
   int k_issued = 0, v_issued = 0;  // producer: tiles whose K / V copies were started
 
-  if (warp == 0) {
+  if (warp < 4) {
+    regs_dec<kRegsLow>();
+    if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
       prefetch_tmap(&p.tmap_q);
@@ -319,9 +342,39 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         record_timeout(p, &abort_flag);
       }
     }
+    }
+    // ---------------------------------------------------------------- teardown (warpgroup 0)
+    __syncwarp();
+    tc_fence_before();
+    __syncthreads();
+    if (abort_flag && lane == 0) {
+      // Some wait expired.  Before the CTA exits, wait (bounded, ignoring
+      // the abort flag) for what this CTA still has in flight: the TMA
+      // copies the producer started (a stage's barrier cannot run ahead of
+      // the last copy started into it) and every MMA the issuer started.
+      const int zero = 0;
+      if (warp == 0) {
+        mbar_wait(&bars.q_full, 0, &zero, tmo);
+        for (int i = (k_issued > C::kKStages ? k_issued - C::kKStages : 0); i < k_issued; ++i)
+          mbar_wait(&bars.k_full[i % C::kKStages], (uint32_t)(i / C::kKStages) & 1u, &zero, tmo);
+        for (int i = (v_issued > C::kVStages ? v_issued - C::kVStages : 0); i < v_issued; ++i) {
+          if (p.fault_mode == 1 && i == 1) continue;  // the copy the test hook withheld
+          mbar_wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u, &zero, tmo);
+        }
+      } else if (warp == 1) {
+        mma_commit(&bars.drain);
+        mbar_wait(&bars.drain, 0, &zero, tmo);
+      }
+    }
+    __syncwarp();
+    if (warp == 1) {
+      tc_fence_after();
+      tmem_dealloc(tbase, C::kTmemCols);
+    }
   } else {
+    regs_inc<kRegsHigh>();
     // ------------------------------------------------------------ softmax + epilogue
-    const int b = (warp - 2) >> 2;                 // query tile of this warpgroup
+    const int b = (warp >> 2) - 1;                 // query tile of this warpgroup
     const int q4 = warp & 3;                       // TMEM lane quarter this warp may access
     const int row = q4 * 32 + lane;                // query row inside the tile
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
@@ -340,37 +393,33 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         tc_fence_after();
         const int t = (t_begin + i) % p.nt_slot;  // key tile inside its slot
         const int valid = (t == p.nt_slot - 1) ? p.valid_last : kTile;
-        float m_tile;
-        {
-          // pass 1: row max over the 128 keys of the tile
-          uint32_t s[4][32];
+        uint32_t s[4][32];
 #pragma unroll
-          for (int c = 0; c < 4; ++c) tmem_ld32(scol + c * 32, s[c]);
+        for (int c = 0; c < 4; ++c) tmem_ld32(scol + c * 32, s[c]);
 #pragma unroll
-          for (int c = 0; c < 4; ++c) tmem_wait_ld(s[c]);
-          if (valid < kTile) {
-#pragma unroll
-            for (int c = 0; c < 4; ++c)
-#pragma unroll
-              for (int e = 0; e < 32; ++e)
-                if (c * 32 + e >= valid) s[c][e] = __float_as_uint(-INFINITY);
-          }
-          float mx[8];
-#pragma unroll
-          for (int k = 0; k < 8; ++k) mx[k] = -INFINITY;
+        for (int c = 0; c < 4; ++c) tmem_wait_ld(s[c]);
+        if (valid < kTile) {
 #pragma unroll
           for (int c = 0; c < 4; ++c)
 #pragma unroll
-            for (int e = 0; e < 32; e += 8) {
-              const int k = (c & 1) * 4 + (e >> 3);
-              mx[k] = max3(mx[k], __uint_as_float(s[c][e]), __uint_as_float(s[c][e + 1]));
-              mx[k] = max3(mx[k], __uint_as_float(s[c][e + 2]), __uint_as_float(s[c][e + 3]));
-              mx[k] = max3(mx[k], __uint_as_float(s[c][e + 4]), __uint_as_float(s[c][e + 5]));
-              mx[k] = max3(mx[k], __uint_as_float(s[c][e + 6]), __uint_as_float(s[c][e + 7]));
-            }
-          m_tile = max3(max3(mx[0], mx[1], mx[2]), max3(mx[3], mx[4], mx[5]),
-                        fmaxf(mx[6], mx[7])) * sl2;
+            for (int e = 0; e < 32; ++e)
+              if (c * 32 + e >= valid) s[c][e] = __float_as_uint(-INFINITY);
         }
+        float mx[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) mx[k] = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < 4; ++c)
+#pragma unroll
+          for (int e = 0; e < 32; e += 8) {
+            const int k = (c & 1) * 4 + (e >> 3);
+            mx[k] = max3(mx[k], __uint_as_float(s[c][e]), __uint_as_float(s[c][e + 1]));
+            mx[k] = max3(mx[k], __uint_as_float(s[c][e + 2]), __uint_as_float(s[c][e + 3]));
+            mx[k] = max3(mx[k], __uint_as_float(s[c][e + 4]), __uint_as_float(s[c][e + 5]));
+            mx[k] = max3(mx[k], __uint_as_float(s[c][e + 6]), __uint_as_float(s[c][e + 7]));
+          }
+        const float m_tile =
+            max3(max3(mx[0], mx[1], mx[2]), max3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])) * sl2;
         const float m_new = fmaxf(m, m_tile);
         const bool need = m_new > m + kRescaleThreshold;
         if (__any_sync(0xffffffffu, need)) {
@@ -394,35 +443,21 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         }
         const uint64_t negm = f2u(-m, -m);
         uint64_t acc[4] = {0, 0, 0, 0};
-        // pass 2: S again, 64 keys at a time; P of 32 keys packs into 16
-        // words written over the first half of the same registers (word e/2
-        // is written after elements e, e+1 are read), then stored over S.
+        // P of 32 keys packs into 16 words, written over the first half of
+        // the same registers (word e/2 is written after elements e, e+1 are
+        // read); two such halves make one 32-column store over S.
 #pragma unroll
-        for (int c2 = 0; c2 < 2; ++c2) {
-          uint32_t s[2][32];
-          tmem_ld32(scol + c2 * 64, s[0]);
-          tmem_ld32(scol + c2 * 64 + 32, s[1]);
-          tmem_wait_ld(s[0]);
-          tmem_wait_ld(s[1]);
-          if (valid < kTile) {
+        for (int c = 0; c < 4; ++c) {
 #pragma unroll
-            for (int cc = 0; cc < 2; ++cc)
-#pragma unroll
-              for (int e = 0; e < 32; ++e)
-                if (c2 * 64 + cc * 32 + e >= valid) s[cc][e] = __float_as_uint(-INFINITY);
+          for (int e = 0; e < 32; e += 2) {
+            float x0, x1;
+            ffma2(x0, x1, __uint_as_float(s[c][e]), __uint_as_float(s[c][e + 1]), sl2x2, negm);
+            const float p0 = ex2(x0);
+            const float p1 = ex2(x1);
+            acc[(e >> 1) & 3] = fadd2(acc[(e >> 1) & 3], p0, p1);
+            s[c][e >> 1] = pack_bf16(p0, p1);
           }
-#pragma unroll
-          for (int cc = 0; cc < 2; ++cc)
-#pragma unroll
-            for (int e = 0; e < 32; e += 2) {
-              float x0, x1;
-              ffma2(x0, x1, __uint_as_float(s[cc][e]), __uint_as_float(s[cc][e + 1]), sl2x2, negm);
-              const float p0 = ex2(x0);
-              const float p1 = ex2(x1);
-              acc[(e >> 1) & 3] = fadd2(acc[(e >> 1) & 3], p0, p1);
-              s[cc][e >> 1] = pack_bf16(p0, p1);
-            }
-          tmem_st32_halves(scol + c2 * 32, s[0], s[1]);
+          if (c & 1) tmem_st32_halves(scol + (c >> 1) * 32, s[c - 1], s[c]);
         }
         float a0, a1, a2, a3, a4, a5, a6, a7;
         u2f(acc[0], a0, a1);
@@ -497,7 +532,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         // wait results were, so none can be left waiting here.
         const uint32_t nsoft = has_q1 ? 256u : 128u;
         asm volatile("bar.sync 1, %0;" ::"r"(nsoft) : "memory");
-        if (threadIdx.x == 64) {
+        if (threadIdx.x == 128) {
           int last = 0;
           if (!abort_flag) last = atomicAdd(&p.ws_count[unit], 1) == p.n_split - 1;
           last_split = last;
@@ -545,39 +580,14 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
             }
             if (lse_at != nullptr) *lse_at = (M + __log2f(L)) * 0.69314718055994531f;
           }
-          if (threadIdx.x == 64) p.ws_count[unit] = 0;  // ready for the next launch
+          if (threadIdx.x == 128) p.ws_count[unit] = 0;  // ready for the next launch
         }
       }
     }
-  }
-
-  // ---------------------------------------------------------------- teardown
-  __syncwarp();
-  tc_fence_before();
-  __syncthreads();
-  if (abort_flag && lane == 0) {
-    // Some wait expired.  Before the CTA exits, wait (bounded, ignoring the
-    // abort flag) for what this CTA still has in flight: the TMA copies the
-    // producer started (a stage's barrier cannot run ahead of the last copy
-    // started into it) and every MMA the issuer started.
-    const int zero = 0;
-    if (warp == 0) {
-      mbar_wait(&bars.q_full, 0, &zero, tmo);
-      for (int i = (k_issued > C::kKStages ? k_issued - C::kKStages : 0); i < k_issued; ++i)
-        mbar_wait(&bars.k_full[i % C::kKStages], (uint32_t)(i / C::kKStages) & 1u, &zero, tmo);
-      for (int i = (v_issued > C::kVStages ? v_issued - C::kVStages : 0); i < v_issued; ++i) {
-        if (p.fault_mode == 1 && i == 1) continue;  // the copy the test hook withheld
-        mbar_wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u, &zero, tmo);
-      }
-    } else if (warp == 1) {
-      mma_commit(&bars.drain);
-      mbar_wait(&bars.drain, 0, &zero, tmo);
-    }
-  }
-  __syncwarp();
-  if (warp == 1) {
-    tc_fence_after();
-    tmem_dealloc(tbase, C::kTmemCols);
+    // ---------------------------------------------------------------- teardown (softmax)
+    __syncwarp();
+    tc_fence_before();
+    __syncthreads();
   }
 }
 
@@ -593,6 +603,14 @@ cudaError_t launch_d(const AttnParams& p, int grid, cudaStream_t s) {
     e = cudaFuncSetAttribute(attend_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              C::kSmemBytes);
     if (e != cudaSuccess) return e;
+    // setmaxnreg.inc waits until the block's register pool can serve it: a
+    // build whose launch register count leaves the split short would never
+    // proceed, so such a build is refused here.
+    cudaFuncAttributes fa;
+    e = cudaFuncGetAttributes(&fa, attend_kernel<D>);
+    if (e != cudaSuccess) return e;
+    if (fa.numRegs * kThreads < 4 * 32 * kRegsLow + 8 * 32 * kRegsHigh)
+      return cudaErrorInvalidConfiguration;
     configured[dev] = true;
   }
   attend_kernel<D><<<grid, kThreads, C::kSmemBytes, s>>>(p);
