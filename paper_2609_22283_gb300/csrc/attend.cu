@@ -72,8 +72,8 @@ __device__ __forceinline__ uint32_t col_o(int b) { return b ? 384u : 256u; }
 // 4*32*kRegsLow + 8*32*kRegsHigh <= 384*kLaunchRegs, checked at launch.
 constexpr int kThreads = 384;
 constexpr int kLaunchRegs = 168;
-constexpr int kRegsLow = 72;
-constexpr int kRegsHigh = 216;
+constexpr int kRegsLow = 88;
+constexpr int kRegsHigh = 208;
 static_assert(4 * 32 * kRegsLow + 8 * 32 * kRegsHigh <= kThreads * kLaunchRegs, "register split");
 constexpr float kRescaleThreshold = 8.0f;  // log2 units: P <= 2^8 between rescales
 
@@ -267,30 +267,38 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     if (lane == 0) {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(128, 128, false);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, true);
-      const uint32_t aQ0 = smem_u32(sQ0);
-      const uint32_t aQ1 = smem_u32(sQ1);
-      const uint32_t aK = smem_u32(sK);
-      const uint32_t aV = smem_u32(sV);
+      // Base descriptors are built once; an MMA's operand descriptor is its
+      // base plus a compile-time offset (the start-address field holds
+      // address >> 4 and every operand lies below 256 KB, so the add never
+      // carries out of the field).  Rebuilding descriptors per MMA costs the
+      // single issuing thread about as long as the MMA itself takes.
+      const uint64_t dQ[2] = {sdesc_sw128(smem_u32(sQ0), 16, 1024),
+                              sdesc_sw128(smem_u32(sQ1), 16, 1024)};
+      const uint64_t dK = sdesc_sw128(smem_u32(sK), 16, 1024);
+      const uint64_t dV = sdesc_sw128(smem_u32(sV), C::kBoxBytes, 1024);
+      constexpr uint64_t kTileStep = (uint64_t)(C::kTileBytes >> 4);
       // S_b = Q_b K_i^T into TMEM buffer b
       auto issue_s = [&](int b, int i) {
-        const uint32_t kb = aK + (i % C::kKStages) * C::kTileBytes;
-        const uint32_t qb = b ? aQ1 : aQ0;
+        const uint64_t kb = dK + (uint64_t)(i % C::kKStages) * kTileStep;
+        const uint64_t qb = dQ[b];
+        const uint32_t dcol = tbase + col_s(b);
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * C::kBoxBytes + (kk & 3) * 32;
-          mma_ss(tbase + col_s(b), sdesc_sw128(qb + off, 16, 1024),
-                 sdesc_sw128(kb + off, 16, 1024), idesc_qk, kk > 0 ? 1u : 0u);
+          const uint64_t off = (uint64_t)(((kk >> 2) * C::kBoxBytes + (kk & 3) * 32) >> 4);
+          mma_ss(dcol, qb + off, kb + off, idesc_qk, kk > 0 ? 1u : 0u);
         }
         mma_commit(&bars.s_full[b]);
       };
       // O_b += P_b V_i with P_b read from TMEM over S_b
       auto issue_pv = [&](int b, int i) {
-        const uint32_t vb = aV + (i % C::kVStages) * C::kTileBytes;
+        const uint64_t vb = dV + (uint64_t)(i % C::kVStages) * kTileStep;
+        const uint32_t ocol = tbase + col_o(b);
+        const uint32_t pcol = tbase + col_s(b);
+        const uint32_t acc0 = i > 0 ? 1u : 0u;
 #pragma unroll
         for (int kk = 0; kk < kTile / 16; ++kk)
-          mma_ts(tbase + col_o(b), tbase + col_s(b) + kk * 8,
-                 sdesc_sw128(vb + kk * 2048, C::kBoxBytes, 1024), idesc_pv,
-                 (i > 0 || kk > 0) ? 1u : 0u);
+          mma_ts(ocol, pcol + kk * 8, vb + (uint64_t)((kk * 2048) >> 4), idesc_pv,
+                 kk > 0 ? 1u : acc0);
       };
       auto wait_k = [&](int i) {
         return mbar_wait(&bars.k_full[i % C::kKStages], (uint32_t)(i / C::kKStages) & 1u,
