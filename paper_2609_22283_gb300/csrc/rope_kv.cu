@@ -8,10 +8,10 @@
 // adjacent head-dimension elements, rotated in fp32 with cos/sin tables that
 // the host computed in fp64 and rounded once to fp32.
 //
-// Bandwidth-bound: every thread owns one 16-byte vector (8 bf16, 4 pairs) of
-// one (node, token, head) row and moves it for K, V and optionally Q, so the
-// position and table work is shared by the three tensors.  Reads walk the
-// token-major inputs linearly; each warp writes two whole 256-byte cache rows.
+// Bandwidth-bound: each warp moves one token's K, V (and Q) rows for all heads
+// as 16-byte vectors, so the position and table work is shared by the heads
+// and the three tensors.  Reads are contiguous per token; every store covers
+// whole 256-byte (or 128-byte) cache rows per half-warp.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -37,60 +37,68 @@ __device__ __forceinline__ uint32_t rotate_pair(uint32_t xy, float c, float s) {
   return *reinterpret_cast<uint32_t*>(&r);
 }
 
+// One warp per (node, token).  A token's H*d values are contiguous in the
+// token-major inputs, so the warp walks them as 16-byte vectors; lane l always
+// holds vector l mod (d/8) of a head row, i.e. the same four pairs for every
+// head, so its cos/sin come from the tables once per token.
 __global__ void __launch_bounds__(256) rope_kv_kernel(const __grid_constant__ RopeParams p) {
+  const int lane = threadIdx.x & 31;
   const int vpr = p.d >> 3;                        // 16-byte vectors per (token, head) row
-  const long long per_node = (long long)p.T * p.H * vpr;
-  const long long total = per_node * p.n_nodes;
+  const int vshift = (vpr == 16) ? 4 : 3;
+  const int c8 = lane & (vpr - 1);
+  const int per_tok = p.H * vpr;                   // vectors per token
   const int HpWp = p.Hp * p.Wp;
   const size_t kv_stride = (size_t)p.H * p.Tpad * p.d;  // elements between K and V of a slot
   const __nv_bfloat16* kin = static_cast<const __nv_bfloat16*>(p.k_new);
   const __nv_bfloat16* vin = static_cast<const __nv_bfloat16*>(p.v_new);
   __nv_bfloat16* qio = static_cast<__nv_bfloat16*>(p.q);
   __nv_bfloat16* cache = static_cast<__nv_bfloat16*>(p.cache);
+  const int warps_per_block = blockDim.x >> 5;
+  const int n_tok = p.n_nodes * p.T;
 
-  for (long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x; idx < total;
-       idx += (long long)gridDim.x * blockDim.x) {
-    const int node = (int)(idx / per_node);
-    const long long rem = idx - (long long)node * per_node;
-    const int c8 = (int)(rem % vpr);
-    const long long rh = rem / vpr;
-    const int h = (int)(rh % p.H);
-    const int u = (int)(rh / p.H);
+  for (int tok = blockIdx.x * warps_per_block + (threadIdx.x >> 5); tok < n_tok;
+       tok += gridDim.x * warps_per_block) {
+    const int node = tok / p.T;
+    const int u = tok - node * p.T;
     const int f = u / HpWp;
     const int hw = u - f * HpWp;
     const int hh = hw / p.Wp;
     const int ww = hw - hh * p.Wp;
     const RopeNode nd = p.nodes[node];
     const int tpos = nd.t_base + f;
-
-    const size_t in_off = (size_t)idx * 8;  // inputs are [node][T][H][d]: linear in idx
-    const uint4 kv = ld_stream(kin + in_off);
-    const uint4 vv = ld_stream(vin + in_off);
-    uint4 qv = make_uint4(0, 0, 0, 0);
-    if (qio) qv = *reinterpret_cast<const uint4*>(qio + in_off);
-
-    uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w};
-    uint32_t qw[4] = {qv.x, qv.y, qv.z, qv.w};
+    float2 cs[4];
 #pragma unroll
     for (int k = 0; k < 4; ++k) {
       const int pi = c8 * 4 + k;  // pair index within the head dimension
-      float2 cs;
-      if (pi < p.P0) {
-        cs = __ldg(p.tab_t + (size_t)tpos * p.P0 + pi);
-      } else if (pi < p.P0 + p.P1) {
-        cs = __ldg(p.tab_h + (size_t)hh * p.P1 + (pi - p.P0));
-      } else {
-        cs = __ldg(p.tab_w + (size_t)ww * p.P2 + (pi - p.P0 - p.P1));
-      }
-      kw[k] = rotate_pair(kw[k], cs.x, cs.y);
-      qw[k] = rotate_pair(qw[k], cs.x, cs.y);
+      if (pi < p.P0)
+        cs[k] = __ldg(p.tab_t + (size_t)tpos * p.P0 + pi);
+      else if (pi < p.P0 + p.P1)
+        cs[k] = __ldg(p.tab_h + (size_t)hh * p.P1 + (pi - p.P0));
+      else
+        cs[k] = __ldg(p.tab_w + (size_t)ww * p.P2 + (pi - p.P0 - p.P1));
     }
-
-    const size_t row = (((size_t)nd.slot * 2) * p.H + h) * p.Tpad + u;
-    __nv_bfloat16* kdst = cache + row * p.d + c8 * 8;
-    *reinterpret_cast<uint4*>(kdst) = make_uint4(kw[0], kw[1], kw[2], kw[3]);
-    *reinterpret_cast<uint4*>(kdst + kv_stride) = vv;
-    if (qio) *reinterpret_cast<uint4*>(qio + in_off) = make_uint4(qw[0], qw[1], qw[2], qw[3]);
+    const size_t in_tok = (size_t)tok * per_tok * 8;
+    const size_t out_slot = ((size_t)nd.slot * 2 * p.H) * p.Tpad;  // row of (slot, K, head 0)
+#pragma unroll 4
+    for (int v = lane; v < per_tok; v += 32) {
+      const int h = v >> vshift;
+      const size_t in_off = in_tok + (size_t)v * 8;
+      const uint4 kv = ld_stream(kin + in_off);
+      const uint4 vv = ld_stream(vin + in_off);
+      uint4 qv = make_uint4(0, 0, 0, 0);
+      if (qio) qv = *reinterpret_cast<const uint4*>(qio + in_off);
+      uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w};
+      uint32_t qw[4] = {qv.x, qv.y, qv.z, qv.w};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        kw[k] = rotate_pair(kw[k], cs[k].x, cs[k].y);
+        qw[k] = rotate_pair(qw[k], cs[k].x, cs[k].y);
+      }
+      __nv_bfloat16* kdst = cache + ((out_slot + (size_t)h * p.Tpad + u) * p.d + c8 * 8);
+      *reinterpret_cast<uint4*>(kdst) = make_uint4(kw[0], kw[1], kw[2], kw[3]);
+      *reinterpret_cast<uint4*>(kdst + kv_stride) = vv;
+      if (qio) *reinterpret_cast<uint4*>(qio + in_off) = make_uint4(qw[0], qw[1], qw[2], qw[3]);
+    }
   }
 }
 
