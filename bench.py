@@ -396,6 +396,71 @@ def run_ours(args, world, rank, local):
     return 0
 
 
+def compare_schedules(args):
+    """Per-chunk attention-layer time of the two executions of Table 3 (Section 5),
+    on one GPU: fully serial clean history (Eq. 5; five one-node launches per
+    chunk: four denoising updates and the clean refresh, W = 6) against the
+    progressive pipeline (one launch of a round's four nodes plus the refresh)."""
+    import torch
+
+    import __graft_entry__
+    from paper_2609_22283_gb300 import inputs as I
+    from paper_2609_22283_gb300.pipeline import Step
+
+    __graft_entry__.build()
+    torch.cuda.set_device(0)
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device="cuda")
+    res = {}
+    for name in ("clean5", "prog4r"):
+        w = I.WORKLOADS[name]
+        inp = I.generate(w)
+        step = Step(w)
+        step.prefill(inp)
+        q, k, v = step.device_inputs(inp)
+        out, lse = step.outputs()
+        nodes, n = step.node_table()
+
+        def one_chunk():
+            if name == "clean5":                        # one launch per node, in order
+                for i in range(n):
+                    sl = slice(i, i + 1)
+                    one = nodes[i:i + 1]
+                    arr = (type(nodes[0]) * 1)(one[0])
+                    step.cache.rope_kv_write(arr, k[sl], v[sl], q[sl], check=False)
+                    step.cache.attend_nodes(arr, q[sl], out[sl], lse[sl], step.scale, check=False)
+            else:
+                step.cache.rope_kv_write(nodes, k, v, q, check=False)
+                step.cache.attend_nodes(nodes, q, out, lse, step.scale, check=False)
+
+        for _ in range(args.warmup):
+            one_chunk()
+        total = 0.0
+        for _ in range(args.steps):
+            flush.zero_()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            one_chunk()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            total += e0.elapsed_time(e1)
+        if step.cache.poll() != 0:
+            raise RuntimeError("device status after timing")
+        res[name] = total / args.steps
+        step.close()
+    line = {"metric": "attention-layer time per chunk (RoPE + cache write + attention), ms",
+            "clean_serial_ms": res["clean5"], "progressive_pipeline_ms": res["prog4r"],
+            "speedup": res["clean5"] / res["prog4r"], "higher_is_better": False,
+            "steps": args.steps, "warmup": args.warmup, "n_gpus": 1, "data": "synthetic",
+            "config": {"serial": I.WORKLOADS["clean5"].description,
+                       "pipeline": I.WORKLOADS["prog4r"].description},
+            "paper_context": "full-DiT steady-state speedup 1.57-2.83x on 4-12 Ascend 910B2C with "
+                             "context parallelism (Table 3); not the same measurement"}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
@@ -406,9 +471,13 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--reference-seconds", type=float, default=8.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--compare-schedules", action="store_true",
+                    help="time clean-serial against progressive-pipeline execution of one chunk")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    if args.compare_schedules:
+        return compare_schedules(args)
     world, rank, local = dist_setup()
     if args.impl == "reference":
         rc = run_reference(args, world, rank)

@@ -102,6 +102,20 @@ WORKLOADS = {
         nodes=_round_nodes(0, 4, 20), prefilled=_PROG_PREFILL_20, round=20,
         description="round 20 of a K=4 pipeline: nodes (20,4),(19,3),(18,2),(17,1), progressive "
                     "history W=6 (7-chunk window, Lkv 32760), in-round reads, 12 heads x 128"),
+    "prog4r": Workload(
+        name="prog4r", seed=5, F=3, Hp=30, Wp=52, H=12, d=128, K=4, W=6, policy="prog",
+        nodes=_round_nodes(0, 4, 20) + ((0, 16, 0),),
+        prefilled=tuple((0, c, 0) for c in range(10, 16)), round=20,
+        description="round 20 of a K=4 progressive pipeline with the clean-state KV refresh of "
+                    "chunk 16 (level 0) in the same launch: 5 nodes, W=6, nodes (17,1) and "
+                    "(20,4) read the refreshed (16,0) in-round, 12 heads x 128"),
+    "clean5": Workload(
+        name="clean5", seed=6, F=3, Hp=30, Wp=52, H=12, d=128, K=4, W=6, policy="clean",
+        nodes=tuple((0, 20, j) for j in range(4, -1, -1)),
+        prefilled=tuple((0, c, 0) for c in range(14, 20)),
+        description="fully serial execution of chunk 20 (Eq. 5): its 4 denoising updates and "
+                    "its clean-state refresh, each a separate one-node launch over 6 clean "
+                    "history chunks (Lkv 32760), 12 heads x 128"),
     "stress14b": Workload(
         name="stress14b", seed=4, F=3, Hp=30, Wp=52, H=40, d=128, K=4, W=6, policy="prog",
         nodes=_round_nodes(0, 4, 20) + _round_nodes(1, 4, 20),
@@ -111,8 +125,10 @@ WORKLOADS = {
                     "N(0,1) with 1% x10 outliers"),
 }
 
-# The order the workloads are listed in the task's configuration table.
+# The order the workloads are listed in the configuration table; prog4r adds
+# the clean-state refresh node to prog4's round.
 ORDER = ("tiny", "clean1", "same4", "prog4", "stress14b")
+EXTRA = ("prog4r", "clean5")
 
 
 @dataclass

@@ -75,7 +75,7 @@ def test_cache_indexing_and_rope(oracle_mod, name):
 
 
 @pytest.mark.parametrize("name,rows_per_head", [("clean1", 48), ("same4", 32), ("prog4", 32),
-                                                ("stress14b", 16)])
+                                                ("prog4r", 24), ("stress14b", 16)])
 def test_full_geometry_sampled(oracle_mod, name, rows_per_head):
     w = I.WORKLOADS[name]
     inp = I.generate(w)

@@ -153,7 +153,7 @@ def test_rows_independent(oracle_mod):
     np.testing.assert_array_equal(pl[0], fl[1][rows])
 
 
-@pytest.mark.parametrize("name", ["clean1", "prog4"])
+@pytest.mark.parametrize("name", ["clean1", "same4", "prog4", "prog4r", "stress14b"])
 def test_full_geometry_selection_is_prefilled(oracle_mod, name):
     """Every state a workload's nodes select is either prefilled or written by
     a node of the same step (the in-round progressive reads)."""
