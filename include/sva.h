@@ -60,6 +60,13 @@ enum {
   SVA_POLICY_PROG = 2   /* phi(j, r) = max(j - r, 0) */
 };
 
+/* Visibility inside a node's own chunk (Eq. 4, Section 3.2: attention within
+ * the current chunk "may be bidirectional"). */
+enum {
+  SVA_WITHIN_BIDIRECTIONAL = 0, /* every own-chunk key visible to every query */
+  SVA_WITHIN_FRAME_CAUSAL = 1   /* a query of latent frame f sees own-chunk keys of frames <= f */
+};
+
 #define SVA_MAX_CTX 16   /* history states one node may read */
 #define SVA_MAX_NODES 64 /* nodes in one sva_rope_kv_write / sva_attend_nodes call */
 
@@ -96,6 +103,8 @@ typedef struct {
  *   chunk, level the node (b, j)
  *   own_slot     cache slot bound to (seq, chunk, level); written by
  *                sva_rope_kv_write, always visible to the node itself
+ *   within       SVA_WITHIN_BIDIRECTIONAL or SVA_WITHIN_FRAME_CAUSAL; the
+ *                history states are always wholly visible
  *   n_ctx        number of history states read, 0..SVA_MAX_CTX
  *   ctx_slot     their cache slots (e.g. from sva_select_context +
  *                sva_cache_lookup), each of a chunk < `chunk`
@@ -106,6 +115,7 @@ typedef struct {
   int32_t chunk;
   int32_t level;
   int32_t own_slot;
+  int32_t within;
   int32_t n_ctx;
   int32_t ctx_slot[SVA_MAX_CTX];
   uint8_t ctx_visible[SVA_MAX_CTX];

@@ -183,7 +183,7 @@ def attend_rows(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float,
 
 def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
                  states: dict, q_raw: np.ndarray, heads, rows, scale: float,
-                 hidden: frozenset = frozenset()):
+                 hidden: frozenset = frozenset(), within: str = "bidirectional"):
     """One denoising node (seq, b, j), computed from raw (pre-RoPE) inputs.
 
     states: {(seq, chunk, level): (K_raw, V_raw)} with arrays [T][H][d] holding
@@ -192,6 +192,9 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
     heads, rows: the (head, query row) pairs to compute are heads x rows.
     hidden: selected (chunk, level) states whose visibility is 0 (their
         tokens get M = -inf); by default every selected state is visible.
+    within: "bidirectional" (every key of the own chunk visible) or
+        "frame_causal" (a query of latent frame f sees the own chunk's keys of
+        frames <= f only); the token-level mask of Eq. 4 either way.
 
     Steps (Section 3.2): select the context states of the node with Eq. 2-3;
     rotate the K of the node's own state and of every selected state and the
@@ -209,6 +212,15 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
     rows = np.asarray(list(rows), dtype=np.int64)
     out = np.empty((len(heads), len(rows), g.d))
     lse = np.empty((len(heads), len(rows)))
+    frame_tokens = g.Hp * g.Wp
+    key_frame = np.arange(g.T) // frame_tokens            # latent frame of own-chunk key v
+    # query rows grouped by the mask they get: one group unless frame-causal
+    if within == "frame_causal":
+        groups = [(f, np.nonzero(rows // frame_tokens == f)[0]) for f in range(g.F)]
+    elif within == "bidirectional":
+        groups = [(None, np.arange(len(rows)))]
+    else:
+        raise ValueError(within)
     for hi, h in enumerate(heads):
         ks, vs, ms = [], [], []
         for (c, lvl) in key_states:
@@ -219,9 +231,14 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
             ms.append(np.full(g.T, -np.inf if masked else 0.0))
         k = np.concatenate(ks)
         v = np.concatenate(vs)
-        m = np.concatenate(ms)
         q = bf16(rope_head(np.asarray(q_raw[:, h, :], dtype=np.float64), b, g))[rows]
-        o, l = attend_rows(q, k, v, scale, m)
-        out[hi] = o
-        lse[hi] = l
+        for f, idx in groups:
+            if len(idx) == 0:
+                continue
+            m = np.concatenate(ms)
+            if f is not None:
+                m[:g.T] = np.where(key_frame > f, -np.inf, m[:g.T])   # own chunk comes first
+            o, l = attend_rows(q[idx], k, v, scale, m)
+            out[hi, idx] = o
+            lse[hi, idx] = l
     return out, lse, sel

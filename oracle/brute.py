@@ -71,12 +71,14 @@ def _rope(x: np.ndarray, chunk: int, F: int, Hp: int, Wp: int, pairs, theta: flo
 
 def brute_forward(policy: str, W: int, F: int, Hp: int, Wp: int, pairs, theta: float,
                   node: tuple[int, int, int], grid: dict, q_raw: np.ndarray,
-                  heads, scale: float, hidden=frozenset()):
+                  heads, scale: float, hidden=frozenset(), frame_causal: bool = False):
     """All query rows of `heads` for node (seq, b, j) against the whole grid.
 
     grid: {(seq, chunk, level): (K_raw, V_raw)} [T][H][d]; it may hold states
     the node must NOT see (other levels, future chunks, other sequences).
     hidden: states whose visibility bit is 0 although the policy selects them.
+    frame_causal: inside the own chunk, query token u sees key token v only if
+    v's latent frame is not after u's.
     Returns (out [len(heads)][T][d], lse [len(heads)][T]).
     """
     seq, b, j = node
@@ -98,10 +100,16 @@ def brute_forward(policy: str, W: int, F: int, Hp: int, Wp: int, pairs, theta: f
         V = np.concatenate(vv)
         M = np.concatenate(mm)
         Q = _bf16_vec(_rope(np.asarray(q_raw[:, h, :], np.float64), b, F, Hp, Wp, pairs, theta))
+        own_start = keys.index((seq, b, j)) * T       # where the own chunk sits in the sequence
         out = np.zeros((T, d))
         lse = np.zeros(T)
         for u in range(T):
-            logits = [scale * float(np.dot(Q[u], K[v])) + M[v] for v in range(K.shape[0])]
+            Mu = M.copy()
+            if frame_causal:
+                for v in range(T):
+                    if v // (Hp * Wp) > u // (Hp * Wp):
+                        Mu[own_start + v] = -np.inf
+            logits = [scale * float(np.dot(Q[u], K[v])) + Mu[v] for v in range(K.shape[0])]
             mx = max(logits)
             w = [math.exp(x - mx) if x != -math.inf else 0.0 for x in logits]
             z = math.fsum(w)

@@ -391,6 +391,10 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       const uint64_t sl2x2 = f2u(sl2, sl2);
       const uint32_t scol = tbase + lane_off + col_s(b);
       const uint32_t ocol = tbase + lane_off + col_o(b);
+      const int frame_causal = nd.frame_causal;
+      // first token of the latent frame after this row's (frame-causal mask)
+      const int frame_end = ((qt0 + b) * kTile + row) / p.frame_tokens * p.frame_tokens +
+                            p.frame_tokens;
       float m = -INFINITY;  // running max of scale*log2(e)*logit (possibly stale by < threshold)
       float l = 0.0f;       // running sum of 2^(x - m)
       bool ok = true;
@@ -400,13 +404,18 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         if (!ok) break;
         tc_fence_after();
         const int t = (t_begin + i) % p.nt_slot;  // key tile inside its slot
-        const int valid = (t == p.nt_slot - 1) ? p.valid_last : kTile;
+        int valid = (t == p.nt_slot - 1) ? p.valid_last : kTile;
+        if (frame_causal && t_begin + i < p.nt_slot) {
+          // own-chunk tile under frame causality: keys up to the end of this
+          // row's latent frame are visible (tile 0, frame 0, always is)
+          valid = min(valid, frame_end - t * kTile);
+        }
         uint32_t s[4][32];
 #pragma unroll
         for (int c = 0; c < 4; ++c) tmem_ld32(scol + c * 32, s[c]);
 #pragma unroll
         for (int c = 0; c < 4; ++c) tmem_wait_ld(s[c]);
-        if (valid < kTile) {
+        if (__any_sync(0xffffffffu, valid < kTile)) {
 #pragma unroll
           for (int c = 0; c < 4; ++c)
 #pragma unroll
@@ -449,7 +458,11 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
           l *= alpha;
           m = m_new;
         }
-        const uint64_t negm = f2u(-m, -m);
+        // m stays -inf while a row has seen no visible key (possible in a key
+        // range that starts past a row's frame under frame causality); its
+        // scores are then all -inf and must give P = 0, not NaN.
+        const float m_sub = (m == -INFINITY) ? 0.0f : m;
+        const uint64_t negm = f2u(-m_sub, -m_sub);
         uint64_t acc[4] = {0, 0, 0, 0};
         // P of 32 keys packs into 16 words, written over the first half of
         // the same registers (word e/2 is written after elements e, e+1 are
@@ -490,7 +503,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       if (p.n_split == 1) {
         if (ok) {
           tc_fence_after();
-          const float inv_l = 1.0f / l;
+          const float inv_l = l > 0.0f ? 1.0f / l : 0.0f;  // a row with no visible key: O = 0
 #pragma unroll
           for (int c = 0; c < D / 32; ++c) {
             uint32_t o[32];
@@ -519,7 +532,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         float* part = p.ws + ((size_t)unit * p.n_split + split) * kItem;
         if (ok) {
           tc_fence_after();
-          const float inv_l = 1.0f / l;
+          const float inv_l = l > 0.0f ? 1.0f / l : 0.0f;  // no visible key in this range
           float4* part4 = reinterpret_cast<float4*>(part);
 #pragma unroll
           for (int c = 0; c < D / 32; ++c) {
@@ -556,14 +569,16 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
             mk[k] = k < p.n_split ? __ldcg(base + k * kItem + D * 256 + r) : -INFINITY;
             M = fmaxf(M, mk[k]);
           }
+          const float M_sub = (M == -INFINITY) ? 0.0f : M;  // every range empty: O = 0
           float L = 0.0f;
 #pragma unroll
           for (int k = 0; k < kMaxSplit; ++k) {
-            wk[k] = k < p.n_split ? __ldcg(base + k * kItem + D * 256 + 256 + r) * ex2(mk[k] - M)
-                                  : 0.0f;
+            wk[k] = k < p.n_split
+                        ? __ldcg(base + k * kItem + D * 256 + 256 + r) * ex2(mk[k] - M_sub)
+                        : 0.0f;
             L += wk[k];
           }
-          const float inv_L = 1.0f / L;
+          const float inv_L = L > 0.0f ? 1.0f / L : 0.0f;
 #pragma unroll
           for (int k = 0; k < kMaxSplit; ++k) wk[k] *= inv_L;
           if (in_range) {

@@ -24,6 +24,7 @@ constexpr int kStatusTimeout = SVA_ERR_DEVICE_TIMEOUT;
 struct AttnNode {
   int32_t q_index;
   int32_t n_kv;
+  int32_t frame_causal;  // own-chunk keys of later latent frames masked
   int32_t slot[1 + SVA_MAX_CTX];
 };
 
@@ -42,6 +43,7 @@ struct alignas(128) AttnParams {
   int32_t n_nodes;
   int32_t nt_slot;      // key tiles per slot = Tpad / kTile
   int32_t valid_last;   // valid key rows in the last tile of a slot
+  int32_t frame_tokens; // tokens per latent frame (Hp * Wp)
   int32_t fault_mode;   // 0 in production; see sva_api.cpp
   int32_t n_split;      // key-range splits per work unit (1 = no split)
   float* ws;            // split partials [unit][split][(d + 2) * 256] fp32, or null

@@ -546,8 +546,11 @@ sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes
     if (st != SVA_OK) return st;
     if (n.n_ctx < 0 || n.n_ctx > SVA_MAX_CTX)
       return fail(SVA_ERR_CAPACITY, "node %d: n_ctx %d outside 0..%d", i, n.n_ctx, SVA_MAX_CTX);
+    if (n.within != SVA_WITHIN_BIDIRECTIONAL && n.within != SVA_WITHIN_FRAME_CAUSAL)
+      return fail(SVA_ERR_INVALID_ARGUMENT, "node %d: unknown within-chunk mode %d", i, n.within);
     sva::AttnNode& a = p.nodes[i];
     a.q_index = i;
+    a.frame_causal = n.within == SVA_WITHIN_FRAME_CAUSAL ? 1 : 0;
     a.slot[0] = n.own_slot;
     int nkv = 1;
     for (int k = 0; k < n.n_ctx; ++k) {
@@ -595,6 +598,7 @@ sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes
   p.n_nodes = n_nodes;
   p.nt_slot = c->L.Tpad / sva::kTile;
   p.valid_last = c->L.T - (p.nt_slot - 1) * sva::kTile;
+  p.frame_tokens = g.grid_h * g.grid_w;
   p.fault_mode = c->fault_mode;
   p.timeout_ns = c->timeout_ns;
   c->fault_mode = 0;
@@ -639,8 +643,11 @@ sva_status sva_attend_nodes_noalloc(sva_cache* c, const sva_node* nodes, int32_t
     if (st != SVA_OK) return st;
     if (n.n_ctx < 0 || n.n_ctx > SVA_MAX_CTX)
       return fail(SVA_ERR_CAPACITY, "node %d: n_ctx %d outside 0..%d", i, n.n_ctx, SVA_MAX_CTX);
+    if (n.within != SVA_WITHIN_BIDIRECTIONAL && n.within != SVA_WITHIN_FRAME_CAUSAL)
+      return fail(SVA_ERR_INVALID_ARGUMENT, "node %d: unknown within-chunk mode %d", i, n.within);
     sva::AttnNode& a = p.nodes[i];
     a.q_index = i;
+    a.frame_causal = n.within == SVA_WITHIN_FRAME_CAUSAL ? 1 : 0;
     a.slot[0] = n.own_slot;
     int nkv = 1;
     for (int k = 0; k < n.n_ctx; ++k) {
@@ -723,6 +730,7 @@ sva_status sva_attend_nodes_noalloc(sva_cache* c, const sva_node* nodes, int32_t
   p.H = g.num_heads;
   p.n_nodes = n_nodes;
   p.valid_last = c->L.T - (p.nt_slot - 1) * sva::kTile;
+  p.frame_tokens = g.grid_h * g.grid_w;
   p.fault_mode = 0;
   p.timeout_ns = c->timeout_ns;
   p.n_split = n_split;

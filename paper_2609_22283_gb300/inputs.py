@@ -46,6 +46,7 @@ class Workload:
     outliers: bool = False
     B: int = 40       # chunks in the video (pipeline length, Eq. 6)
     round: int | None = None  # pipeline round the nodes form (Eq. 6), if any
+    within: str = "bidirectional"  # visibility inside the own chunk (or "frame_causal")
     description: str = ""
     theta: float = 10000.0
     pairs: tuple = field(default=None)
@@ -116,6 +117,18 @@ WORKLOADS = {
         description="fully serial execution of chunk 20 (Eq. 5): its 4 denoising updates and "
                     "its clean-state refresh, each a separate one-node launch over 6 clean "
                     "history chunks (Lkv 32760), 12 heads x 128"),
+    "tinyfc": Workload(
+        name="tinyfc", seed=7, F=3, Hp=4, Wp=8, H=2, d=64, K=2, W=2, policy="prog",
+        nodes=((0, 3, 2), (0, 2, 1)), prefilled=((0, 1, 0),), B=3, round=3,
+        within="frame_causal",
+        description="tiny with 3 latent frames of 4x8 tokens per chunk (T=96) and a "
+                    "frame-causal mask inside each own chunk"),
+    "prog4fc": Workload(
+        name="prog4fc", seed=8, F=3, Hp=30, Wp=52, H=12, d=128, K=4, W=6, policy="prog",
+        nodes=_round_nodes(0, 4, 20), prefilled=_PROG_PREFILL_20, round=20,
+        within="frame_causal",
+        description="prog4 with a frame-causal mask inside each own chunk (frames of 1560 "
+                    "tokens, boundaries inside 128-token tiles)"),
     "stress14b": Workload(
         name="stress14b", seed=4, F=3, Hp=30, Wp=52, H=40, d=128, K=4, W=6, policy="prog",
         nodes=_round_nodes(0, 4, 20) + _round_nodes(1, 4, 20),
@@ -128,7 +141,7 @@ WORKLOADS = {
 # The order the workloads are listed in the configuration table; prog4r adds
 # the clean-state refresh node to prog4's round.
 ORDER = ("tiny", "clean1", "same4", "prog4", "stress14b")
-EXTRA = ("prog4r", "clean5")
+EXTRA = ("prog4r", "clean5", "tinyfc", "prog4fc")
 
 
 @dataclass

@@ -67,7 +67,8 @@ class Step:
                 if st != sva.OK:
                     raise sva.SvaError(st, sva.last_error())
             ctx = [self.cache.lookup(s, c, l) for (c, l) in sel]
-            entries.append(dict(seq=s, chunk=b, level=j, own_slot=self.own[(s, b, j)], ctx=ctx))
+            entries.append(dict(seq=s, chunk=b, level=j, own_slot=self.own[(s, b, j)], ctx=ctx,
+                                within=sva.WITHIN[w.within]))
         return sva.make_nodes(entries), len(entries)
 
     def run(self, q, k_new, v_new, out, lse=None, stream=None, rotate_q: bool = True):

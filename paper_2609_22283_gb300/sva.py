@@ -29,6 +29,8 @@ STATUS_NAMES = {0: "OK", 1: "INVALID_ARGUMENT", 2: "NOT_RESIDENT", 3: "CAUSALITY
                 5: "UNSUPPORTED", 6: "CUDA", 7: "DEVICE_TIMEOUT", 8: "UNAVAILABLE"}
 
 POLICY_CLEAN, POLICY_SAME, POLICY_PROG = 0, 1, 2
+WITHIN_BIDIRECTIONAL, WITHIN_FRAME_CAUSAL = 0, 1
+WITHIN = {"bidirectional": WITHIN_BIDIRECTIONAL, "frame_causal": WITHIN_FRAME_CAUSAL}
 POLICIES = {"clean": POLICY_CLEAN, "same": POLICY_SAME, "prog": POLICY_PROG}
 MAX_CTX = 16
 MAX_NODES = 64
@@ -55,7 +57,8 @@ class sva_geometry(ctypes.Structure):
 
 class sva_node(ctypes.Structure):
     _fields_ = [("seq", ctypes.c_int32), ("chunk", ctypes.c_int32), ("level", ctypes.c_int32),
-                ("own_slot", ctypes.c_int32), ("n_ctx", ctypes.c_int32),
+                ("own_slot", ctypes.c_int32), ("within", ctypes.c_int32),
+                ("n_ctx", ctypes.c_int32),
                 ("ctx_slot", ctypes.c_int32 * MAX_CTX), ("ctx_visible", ctypes.c_uint8 * MAX_CTX)]
 
 
@@ -169,12 +172,13 @@ def cache_bytes(g: sva_geometry) -> int:
 
 def make_nodes(entries) -> ctypes.Array:
     """entries: iterable of dicts with seq, chunk, level, own_slot, ctx (list of slots),
-    visible (optional list of 0/1)."""
+    visible (optional list of 0/1), within (optional, default bidirectional)."""
     entries = list(entries)
     arr = (sva_node * max(len(entries), 1))()
     for i, e in enumerate(entries):
         n = arr[i]
         n.seq, n.chunk, n.level, n.own_slot = e["seq"], e["chunk"], e["level"], e["own_slot"]
+        n.within = e.get("within", WITHIN_BIDIRECTIONAL)
         ctx = list(e.get("ctx", []))
         vis = list(e.get("visible", [1] * len(ctx)))
         n.n_ctx = len(ctx)

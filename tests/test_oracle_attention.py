@@ -162,3 +162,40 @@ def test_full_geometry_selection_is_prefilled(oracle_mod, name):
     for (s, b, j) in w.nodes:
         for (c, lvl) in oracle_mod.select(oracle_mod.POLICY_IDS[w.policy], w.W, b, j):
             assert (s, c, lvl) in have
+
+
+def test_frame_causal_against_dense_brute_force(oracle_mod):
+    from oracle import brute
+    w = I.WORKLOADS["tinyfc"]                 # 3 latent frames of 32 tokens per chunk
+    inp = I.generate(w)
+    g = oracle_mod.Geometry(F=w.F, Hp=w.Hp, Wp=w.Wp, H=w.H, d=w.d, pairs=w.pairs, theta=w.theta)
+    states = {k: (_f64(a), _f64(b)) for k, (a, b) in I.all_states(w, inp).items()}
+    rng = np.random.default_rng(11)
+    grid = dict(states)
+    for s in [(0, 2, 0), (0, 4, 0), (0, 1, 1)]:
+        grid[s] = (rng.standard_normal((w.T, w.H, w.d)), rng.standard_normal((w.T, w.H, w.d)))
+    scale = 1.0 / math.sqrt(w.d)
+    for i, node in enumerate(w.nodes):
+        q = _f64(inp.q[i])
+        out, lse, _ = oracle_mod.node_forward(g, oracle_mod.POLICY_IDS[w.policy], w.W, node, states,
+                                              q, range(w.H), range(w.T), scale, within="frame_causal")
+        bo, bl = brute.brute_forward(w.policy, w.W, w.F, w.Hp, w.Wp, w.pairs, w.theta, node, grid, q,
+                                     range(w.H), scale, frame_causal=True)
+        np.testing.assert_allclose(out, bo, rtol=0, atol=1e-12)
+        np.testing.assert_allclose(lse, bl, rtol=0, atol=1e-12)
+        bid, _, _ = oracle_mod.node_forward(g, oracle_mod.POLICY_IDS[w.policy], w.W, node, states,
+                                            q, range(w.H), range(w.T), scale)
+        last = slice(2 * w.Hp * w.Wp, w.T)    # the last frame sees the whole chunk either way
+        np.testing.assert_array_equal(out[:, last], bid[:, last])
+        assert not np.allclose(out[:, :w.Hp * w.Wp], bid[:, :w.Hp * w.Wp])
+
+
+def test_frame_causal_single_frame_is_bidirectional(oracle_mod):
+    w, inp, g = _tiny(oracle_mod)              # F = 1
+    states = {k: (_f64(a), _f64(b)) for k, (a, b) in I.all_states(w, inp).items()}
+    q = _f64(inp.q[0])
+    a, la, _ = oracle_mod.node_forward(g, 2, w.W, w.nodes[0], states, q, [0, 1], range(w.T), 0.125,
+                                       within="frame_causal")
+    b, lb, _ = oracle_mod.node_forward(g, 2, w.W, w.nodes[0], states, q, [0, 1], range(w.T), 0.125)
+    np.testing.assert_array_equal(a, b)
+    np.testing.assert_array_equal(la, lb)
