@@ -183,6 +183,21 @@ sva_status sva_check_pipeline(int32_t K, int32_t level, int32_t chunk, int32_t n
 sva_status sva_rope_kv_write(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
                              const void* k_new, const void* v_new, void* q_inout, sva_stream s);
 
+/* sva_rope_kv_write with an RMS normalisation of each token's key (and query)
+ * vector in front of the rotation, fused in the same pass (reading: the paper
+ * names no normalisation; Wan-style DiTs normalise q and k this way before
+ * RoPE).  For a token's K row x of H*d elements:
+ *   x' = x * gamma_k / sqrt(mean(x^2) + eps),
+ * then RoPE; likewise Q with gamma_q; V is copied unchanged.  fp32 arithmetic,
+ * one bf16 rounding of the rotated result.
+ *   gamma_k, gamma_q: fp32 [H*d] device vectors, 16-byte aligned (gamma_q may
+ *   be NULL when q_inout is NULL); eps > 0.
+ * Errors: as sva_rope_kv_write, plus INVALID_ARGUMENT for bad gammas or eps. */
+sva_status sva_rope_kv_write_qknorm(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
+                                    const void* k_new, const void* v_new, void* q_inout,
+                                    const float* gamma_k, const float* gamma_q, float eps,
+                                    sva_stream s);
+
 /* Policy-indexed chunk-causal attention (Eq. 4) for a batch of nodes:
  *   out[i][u][h] = sum_v softmax_v(scale * q[i][u][h] . k_v + M(u, v)) v_v
  * over the keys of node i's own slot and its visible context slots; M is 0

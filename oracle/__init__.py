@@ -75,6 +75,8 @@ def _load():
     lib.oracle_bf16_array.restype = None
     lib.oracle_rope_head.argtypes = [pd, pd, i32, i32, i32, i32, i32, lng, pi32, dbl]
     lib.oracle_rope_head.restype = None
+    lib.oracle_rms_norm.argtypes = [pd, pd, pd, lng, i32, dbl]
+    lib.oracle_rms_norm.restype = None
     lib.oracle_attend_rows.argtypes = [pd, pd, pd, pd, lng, i32, lng, dbl, pd, pd]
     lib.oracle_attend_rows.restype = None
     lib.oracle_num_threads.argtypes = []
@@ -158,6 +160,17 @@ def rope_head(x: np.ndarray, b: int, g: Geometry) -> np.ndarray:
     return y
 
 
+def rms_norm(x: np.ndarray, gamma: np.ndarray, eps: float) -> np.ndarray:
+    """RMSNorm of each token's vector: x [T][H][d] (or [T][n]) with gamma [H*d]."""
+    shape = x.shape
+    x2 = np.ascontiguousarray(np.asarray(x, dtype=np.float64).reshape(shape[0], -1))
+    g = np.ascontiguousarray(np.asarray(gamma, dtype=np.float64).reshape(-1))
+    assert g.shape[0] == x2.shape[1]
+    y = np.empty_like(x2)
+    _load().oracle_rms_norm(_pd(x2), _pd(g), _pd(y), x2.shape[0], x2.shape[1], float(eps))
+    return y.reshape(shape)
+
+
 # ---------------------------------------------------------------- attention
 
 def attend_rows(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float,
@@ -183,7 +196,8 @@ def attend_rows(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float,
 
 def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
                  states: dict, q_raw: np.ndarray, heads, rows, scale: float,
-                 hidden: frozenset = frozenset(), within: str = "bidirectional"):
+                 hidden: frozenset = frozenset(), within: str = "bidirectional",
+                 norm=None):
     """One denoising node (seq, b, j), computed from raw (pre-RoPE) inputs.
 
     states: {(seq, chunk, level): (K_raw, V_raw)} with arrays [T][H][d] holding
@@ -195,6 +209,8 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
     within: "bidirectional" (every key of the own chunk visible) or
         "frame_causal" (a query of latent frame f sees the own chunk's keys of
         frames <= f only); the token-level mask of Eq. 4 either way.
+    norm: None, or (gamma_k, gamma_q, eps): every key state's K and the
+        node's Q are RMS-normalised per token (rms_norm) before the rotation.
 
     Steps (Section 3.2): select the context states of the node with Eq. 2-3;
     rotate the K of the node's own state and of every selected state and the
@@ -221,6 +237,11 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
         groups = [(None, np.arange(len(rows)))]
     else:
         raise ValueError(within)
+    if norm is not None:
+        gk, gq, eps = norm
+        states = {s: (rms_norm(states[s][0], gk, eps), states[s][1])
+                  for s in [(seq, c, lvl) for (c, lvl) in key_states]}
+        q_raw = rms_norm(q_raw, gq, eps)
     for hi, h in enumerate(heads):
         ks, vs, ms = [], [], []
         for (c, lvl) in key_states:

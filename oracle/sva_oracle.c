@@ -146,6 +146,19 @@ void oracle_rope_head(const double* x, double* y, int T, int d, int F, int Hp, i
   }
 }
 
+/* RMS normalisation of each row of x[T][n] (reading: the paper names no
+ * normalisation; a token's whole query or key vector of n = H*d elements is
+ * normalised before RoPE): y = x * gamma / sqrt(mean(x^2) + eps), fp64. */
+void oracle_rms_norm(const double* x, const double* gamma, double* y, long T, int n, double eps) {
+  for (long t = 0; t < T; ++t) {
+    const double* xr = x + t * n;
+    double ss = 0.0;
+    for (int i = 0; i < n; ++i) ss += xr[i] * xr[i];
+    const double r = 1.0 / sqrt(ss / n + eps);
+    for (int i = 0; i < n; ++i) y[t * n + i] = xr[i] * r * gamma[i];
+  }
+}
+
 /* Eq. 4 (Section 3.2): masked softmax attention.  For each query row i the
  * logits are l_v = scale * <q_i, k_v> + mask[v], with mask[v] = 0 where the
  * query may attend to key v and -inf otherwise; the mask is added before

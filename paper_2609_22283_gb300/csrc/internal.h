@@ -68,6 +68,11 @@ struct RopeParams {
   int32_t T, H, d, Tpad, Hp, Wp, P0, P1, P2;
   int32_t n_nodes;
   int32_t grid_blocks;
+  // Optional RMSNorm of each token's K (and Q) vector of H*d elements before
+  // the rotation: x * gamma / sqrt(mean(x^2) + eps).  Null gammas: no norm.
+  const float* gamma_k;
+  const float* gamma_q;
+  float norm_eps;
   RopeNode nodes[SVA_MAX_NODES];
 };
 

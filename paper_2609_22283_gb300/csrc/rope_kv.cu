@@ -28,6 +28,32 @@ __device__ __forceinline__ uint4 ld_stream(const void* p) {
   return v;
 }
 
+__device__ __forceinline__ uint32_t rotate_pair_f(float x, float y, float c, float s) {
+  const float rx = __fmaf_rn(x, c, -(y * s));
+  const float ry = __fmaf_rn(x, s, y * c);
+  __nv_bfloat162 r = __floats2bfloat162_rn(rx, ry);  // .x (rx) in the low half
+  return *reinterpret_cast<uint32_t*>(&r);
+}
+
+// bf16 pair (element 2k in the low half) times g0, g1, then rotated
+__device__ __forceinline__ uint32_t norm_rotate_pair(uint32_t xy, float g0, float g1, float c,
+                                                     float s) {
+  return rotate_pair_f(__uint_as_float(xy << 16) * g0, __uint_as_float(xy & 0xFFFF0000u) * g1, c,
+                       s);
+}
+
+__device__ __forceinline__ float sumsq8(uint4 v) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  float a = 0.0f;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const float x = __uint_as_float(w[k] << 16), y = __uint_as_float(w[k] & 0xFFFF0000u);
+    a = __fmaf_rn(x, x, a);
+    a = __fmaf_rn(y, y, a);
+  }
+  return a;
+}
+
 __device__ __forceinline__ uint32_t rotate_pair(uint32_t xy, float c, float s) {
   const float x = __uint_as_float(xy << 16);
   const float y = __uint_as_float(xy & 0xFFFF0000u);
@@ -79,6 +105,26 @@ __global__ void __launch_bounds__(256) rope_kv_kernel(const __grid_constant__ Ro
     }
     const size_t in_tok = (size_t)tok * per_tok * 8;
     const size_t out_slot = ((size_t)nd.slot * 2 * p.H) * p.Tpad;  // row of (slot, K, head 0)
+    // RMSNorm scale of the token's K and Q vectors (pass over the row, then a
+    // warp reduction); the second pass below reloads the row from L1/L2.
+    float rk = 1.0f, rq = 1.0f;
+    const bool norm = p.gamma_k != nullptr;
+    if (norm) {
+      float sk = 0.0f, sq = 0.0f;
+      for (int v = lane; v < per_tok; v += 32) {
+        const size_t off = in_tok + (size_t)v * 8;
+        sk += sumsq8(*reinterpret_cast<const uint4*>(kin + off));
+        if (qio) sq += sumsq8(*reinterpret_cast<const uint4*>(qio + off));
+      }
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        sk += __shfl_xor_sync(0xffffffffu, sk, o);
+        sq += __shfl_xor_sync(0xffffffffu, sq, o);
+      }
+      const float inv_n = 1.0f / (float)(per_tok * 8);
+      rk = __frsqrt_rn(__fmaf_rn(sk, inv_n, p.norm_eps));
+      rq = __frsqrt_rn(__fmaf_rn(sq, inv_n, p.norm_eps));
+    }
 #pragma unroll 4
     for (int v = lane; v < per_tok; v += 32) {
       const int h = v >> vshift;
@@ -89,10 +135,28 @@ __global__ void __launch_bounds__(256) rope_kv_kernel(const __grid_constant__ Ro
       if (qio) qv = *reinterpret_cast<const uint4*>(qio + in_off);
       uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w};
       uint32_t qw[4] = {qv.x, qv.y, qv.z, qv.w};
+      if (norm) {
+        const float4* gk = reinterpret_cast<const float4*>(p.gamma_k + (size_t)v * 8);
+        const float4 gk0 = __ldg(gk), gk1 = __ldg(gk + 1);
+        const float gkk[8] = {gk0.x, gk0.y, gk0.z, gk0.w, gk1.x, gk1.y, gk1.z, gk1.w};
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
-        kw[k] = rotate_pair(kw[k], cs[k].x, cs[k].y);
-        qw[k] = rotate_pair(qw[k], cs[k].x, cs[k].y);
+        for (int k = 0; k < 4; ++k)
+          kw[k] = norm_rotate_pair(kw[k], gkk[2 * k] * rk, gkk[2 * k + 1] * rk, cs[k].x, cs[k].y);
+        if (qio) {
+          const float4* gq = reinterpret_cast<const float4*>(p.gamma_q + (size_t)v * 8);
+          const float4 gq0 = __ldg(gq), gq1 = __ldg(gq + 1);
+          const float gqq[8] = {gq0.x, gq0.y, gq0.z, gq0.w, gq1.x, gq1.y, gq1.z, gq1.w};
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            qw[k] = norm_rotate_pair(qw[k], gqq[2 * k] * rq, gqq[2 * k + 1] * rq, cs[k].x,
+                                     cs[k].y);
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          kw[k] = rotate_pair(kw[k], cs[k].x, cs[k].y);
+          qw[k] = rotate_pair(qw[k], cs[k].x, cs[k].y);
+        }
       }
       __nv_bfloat16* kdst = cache + ((out_slot + (size_t)h * p.Tpad + u) * p.d + c8 * 8);
       *reinterpret_cast<uint4*>(kdst) = make_uint4(kw[0], kw[1], kw[2], kw[3]);

@@ -468,8 +468,14 @@ sva_status sva_check_pipeline(int32_t K, int32_t level, int32_t chunk, int32_t n
   return ok();
 }
 
-sva_status sva_rope_kv_write(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
-                             const void* k_new, const void* v_new, void* q_inout, sva_stream s) {
+}  // extern "C"
+
+namespace {
+
+// sva_rope_kv_write and sva_rope_kv_write_qknorm: gamma_k == NULL means no norm.
+sva_status rope_write(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* k_new,
+                      const void* v_new, void* q_inout, const float* gamma_k,
+                      const float* gamma_q, float eps, sva_stream s) {
   if (c == nullptr || nodes == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "NULL argument");
   if (n_nodes < 1) return fail(SVA_ERR_INVALID_ARGUMENT, "n_nodes %d < 1", n_nodes);
   if (n_nodes > SVA_MAX_NODES)
@@ -514,6 +520,9 @@ sva_status sva_rope_kv_write(sva_cache* c, const sva_node* nodes, int32_t n_node
   p.P1 = g.rope_pairs[1];
   p.P2 = g.rope_pairs[2];
   p.n_nodes = n_nodes;
+  p.gamma_k = gamma_k;
+  p.gamma_q = gamma_k != nullptr && q_inout != nullptr ? gamma_q : nullptr;
+  p.norm_eps = eps;
   const long long tokens = (long long)n_nodes * p.T;  // one warp per token, 8 warps per block
   const long long blocks = (tokens + 7) / 8;
   p.grid_blocks = (int)std::min<long long>(blocks, (long long)c->num_sms * 16);
@@ -521,6 +530,28 @@ sva_status sva_rope_kv_write(sva_cache* c, const sva_node* nodes, int32_t n_node
   if (e != cudaSuccess) return cuda_fail(e, "rope_kv launch");
   for (int i = 0; i < n_nodes; ++i) c->slots[nodes[i].own_slot].resident = true;
   return ok();
+}
+
+}  // namespace
+
+extern "C" {
+
+sva_status sva_rope_kv_write(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
+                             const void* k_new, const void* v_new, void* q_inout, sva_stream s) {
+  return rope_write(c, nodes, n_nodes, k_new, v_new, q_inout, nullptr, nullptr, 0.0f, s);
+}
+
+sva_status sva_rope_kv_write_qknorm(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
+                                    const void* k_new, const void* v_new, void* q_inout,
+                                    const float* gamma_k, const float* gamma_q, float eps,
+                                    sva_stream s) {
+  if (gamma_k == nullptr || !aligned16(gamma_k) ||
+      (q_inout != nullptr && (gamma_q == nullptr || !aligned16(gamma_q))))
+    return fail(SVA_ERR_INVALID_ARGUMENT,
+                "gamma_k (and gamma_q when q_inout is given) must be non-NULL and 16-byte aligned");
+  if (!std::isfinite(eps) || !(eps > 0.0f))
+    return fail(SVA_ERR_INVALID_ARGUMENT, "eps must be finite and > 0");
+  return rope_write(c, nodes, n_nodes, k_new, v_new, q_inout, gamma_k, gamma_q, eps, s);
 }
 
 sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* q,

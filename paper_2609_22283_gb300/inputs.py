@@ -47,6 +47,7 @@ class Workload:
     B: int = 40       # chunks in the video (pipeline length, Eq. 6)
     round: int | None = None  # pipeline round the nodes form (Eq. 6), if any
     within: str = "bidirectional"  # visibility inside the own chunk (or "frame_causal")
+    qknorm: bool = False  # RMS-normalise K and Q per token before RoPE (seeded gammas)
     description: str = ""
     theta: float = 10000.0
     pairs: tuple = field(default=None)
@@ -123,6 +124,10 @@ WORKLOADS = {
         within="frame_causal",
         description="tiny with 3 latent frames of 4x8 tokens per chunk (T=96) and a "
                     "frame-causal mask inside each own chunk"),
+    "tinyn": Workload(
+        name="tinyn", seed=10, F=1, Hp=8, Wp=8, H=2, d=64, K=2, W=2, policy="prog",
+        nodes=((0, 3, 2), (0, 2, 1)), prefilled=((0, 1, 0),), B=3, round=3, qknorm=True,
+        description="tiny with K and Q RMS-normalised per token before RoPE"),
     "prog4fc": Workload(
         name="prog4fc", seed=8, F=3, Hp=30, Wp=52, H=12, d=128, K=4, W=6, policy="prog",
         nodes=_round_nodes(0, 4, 20), prefilled=_PROG_PREFILL_20, round=20,
@@ -141,7 +146,7 @@ WORKLOADS = {
 # The order the workloads are listed in the configuration table; prog4r adds
 # the clean-state refresh node to prog4's round.
 ORDER = ("tiny", "clean1", "same4", "prog4", "stress14b")
-EXTRA = ("prog4r", "clean5", "tinyfc", "prog4fc")
+EXTRA = ("prog4r", "clean5", "tinyfc", "prog4fc", "tinyn")
 
 
 @dataclass
@@ -150,6 +155,9 @@ class Inputs:
     q: torch.Tensor    # bf16 [n][T][H][d]
     k_new: torch.Tensor
     v_new: torch.Tensor
+    gamma_k: torch.Tensor | None = None   # fp32 [H*d], with qknorm
+    gamma_q: torch.Tensor | None = None
+    norm_eps: float = 1e-6
 
 
 def generate(w: Workload) -> Inputs:
@@ -172,7 +180,11 @@ def generate(w: Workload) -> Inputs:
     q = draw((n, T, H, d))
     k_new = draw((n, T, H, d))
     v_new = draw((n, T, H, d))
-    return Inputs(history, q, k_new, v_new)
+    inp = Inputs(history, q, k_new, v_new)
+    if w.qknorm:   # drawn last, so the other tensors match the unnormalised workload
+        inp.gamma_k = torch.rand(H * d, generator=g, dtype=torch.float32) + 0.5
+        inp.gamma_q = torch.rand(H * d, generator=g, dtype=torch.float32) + 0.5
+    return inp
 
 
 def all_states(w: Workload, inp: Inputs) -> dict:

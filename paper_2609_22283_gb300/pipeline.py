@@ -43,6 +43,9 @@ class Step:
     def prefill(self, inp: Inputs, stream=None):
         """Binds and writes the workload's history states (untimed set-up)."""
         w = self.w
+        self.norm = None
+        if w.qknorm:
+            self.norm = (inp.gamma_k.to(self.device), inp.gamma_q.to(self.device), inp.norm_eps)
         pre = list(w.prefilled)
         for start in range(0, len(pre), sva.MAX_NODES):
             group = pre[start:start + sva.MAX_NODES]
@@ -52,7 +55,11 @@ class Step:
                 entries.append(dict(seq=s, chunk=c, level=l, own_slot=slot))
             k = torch.stack([inp.history[tuple(st)][0] for st in group]).to(self.device)
             v = torch.stack([inp.history[tuple(st)][1] for st in group]).to(self.device)
-            self.cache.rope_kv_write(entries, k, v, None, stream=stream)
+            if self.norm is not None:
+                self.cache.rope_kv_write_qknorm(entries, k, v, None, self.norm[0], None,
+                                                self.norm[2], stream=stream)
+            else:
+                self.cache.rope_kv_write(entries, k, v, None, stream=stream)
         for st in w.nodes:
             self.own[tuple(st)] = self.cache.bind(*st)
 
@@ -74,8 +81,13 @@ class Step:
     def run(self, q, k_new, v_new, out, lse=None, stream=None, rotate_q: bool = True):
         """One pass of the hot path on device tensors [n][T][H][d] (q rotated in place)."""
         nodes, n = self.node_table()
-        self.cache.rope_kv_write(nodes, k_new, v_new, q if rotate_q else None, stream=stream,
-                                 check=False)
+        if self.norm is not None:
+            self.cache.rope_kv_write_qknorm(nodes, k_new, v_new, q if rotate_q else None,
+                                            self.norm[0], self.norm[1], self.norm[2],
+                                            stream=stream)
+        else:
+            self.cache.rope_kv_write(nodes, k_new, v_new, q if rotate_q else None, stream=stream,
+                                     check=False)
         self.cache.attend_nodes(nodes, q, out, lse, self.scale, stream=stream, check=False)
         return n
 

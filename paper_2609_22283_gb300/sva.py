@@ -37,7 +37,8 @@ MAX_NODES = 64
 
 EXPORTED = ("sva_cache_bytes", "sva_cache_create", "sva_cache_bind", "sva_cache_lookup",
             "sva_cache_release", "sva_select_context", "sva_pipeline_round", "sva_check_pipeline",
-            "sva_rope_kv_write", "sva_attend_nodes", "sva_attend_workspace_bytes",
+            "sva_rope_kv_write", "sva_rope_kv_write_qknorm", "sva_attend_nodes",
+            "sva_attend_workspace_bytes",
             "sva_cache_set_workspace", "sva_attend_nodes_noalloc", "sva_poll_device_status",
             "sva_debug_inject", "sva_destroy", "sva_last_error")
 
@@ -87,6 +88,7 @@ def load(path: str = LIB_PATH):
         "sva_pipeline_round": ([i32, i32, i32, i32, pi32, pi32, pi32], i32),
         "sva_check_pipeline": ([i32, i32, i32, i32, pi32, pi32], i32),
         "sva_rope_kv_write": ([p, pn, i32, p, p, p, p], i32),
+        "sva_rope_kv_write_qknorm": ([p, pn, i32, p, p, p, p, p, ctypes.c_float, p], i32),
         "sva_attend_nodes": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
         "sva_attend_workspace_bytes": ([p], ctypes.c_size_t),
         "sva_attend_nodes_noalloc": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
@@ -244,6 +246,22 @@ class Cache:
                                     ctypes.c_void_p(v_new.data_ptr()),
                                     ctypes.c_void_p(q.data_ptr() if q is not None else 0),
                                     ctypes.c_void_p(_stream_handle(stream)))
+        _check(st)
+
+    def rope_kv_write_qknorm(self, nodes, k_new, v_new, q, gamma_k, gamma_q, eps=1e-6,
+                             stream=None):
+        """sva_rope_kv_write_qknorm: RMSNorm (fp32 gammas of H*d) then RoPE."""
+        arr = nodes if isinstance(nodes, ctypes.Array) else make_nodes(nodes)
+        for gname, gm in (("gamma_k", gamma_k), ("gamma_q", gamma_q)):
+            if gm is not None and (gm.dtype != torch.float32 or not gm.is_cuda
+                                   or not gm.is_contiguous()):
+                raise ValueError(f"{gname} must be a contiguous fp32 CUDA tensor")
+        st = _lib.sva_rope_kv_write_qknorm(
+            self.handle, arr, len(arr), ctypes.c_void_p(k_new.data_ptr()),
+            ctypes.c_void_p(v_new.data_ptr()), ctypes.c_void_p(q.data_ptr() if q is not None else 0),
+            ctypes.c_void_p(gamma_k.data_ptr()),
+            ctypes.c_void_p(gamma_q.data_ptr() if gamma_q is not None else 0), float(eps),
+            ctypes.c_void_p(_stream_handle(stream)))
         _check(st)
 
     def attend_nodes(self, nodes, q, out, lse=None, scale=None, stream=None, check=True):

@@ -32,7 +32,9 @@ def oracle_node(w, inp, states, node_index, heads, rows, hidden=frozenset()):
     q = inp.q[node_index].to(torch.float64).numpy()
     out, lse, _ = oracle.node_forward(g, oracle.POLICY_IDS[w.policy], w.W, w.nodes[node_index],
                                       states, q, list(heads), list(rows), 1.0 / math.sqrt(w.d),
-                                      hidden=hidden, within=w.within)
+                                      hidden=hidden, within=w.within,
+                                      norm=((inp.gamma_k.double().numpy(), inp.gamma_q.double().numpy(),
+                                             inp.norm_eps) if w.qknorm else None))
     return out, lse
 
 

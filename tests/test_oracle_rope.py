@@ -133,3 +133,16 @@ def test_bf16_rounding_matches_library(oracle_mod):
     lib = torch.from_numpy(x32).to(torch.bfloat16).to(torch.float64).numpy()
     mine = oracle_mod.bf16(x32.astype(np.float64))
     np.testing.assert_array_equal(mine, lib)
+
+
+def test_rms_norm_matches_library(oracle_mod):
+    rng = np.random.default_rng(21)
+    x = rng.standard_normal((40, 3, 16)) * rng.uniform(0.1, 10.0, (40, 1, 1))
+    gamma = rng.uniform(0.5, 1.5, 48)
+    y = oracle_mod.rms_norm(x, gamma, 1e-6)
+    ref = torch.nn.functional.rms_norm(torch.from_numpy(x.reshape(40, 48)), (48,),
+                                       torch.from_numpy(gamma), eps=1e-6).numpy()
+    np.testing.assert_allclose(y.reshape(40, 48), ref, rtol=1e-13, atol=1e-14)
+    # scale invariance (up to eps) and unit RMS with unit gamma
+    y2 = oracle_mod.rms_norm(x * 7.0, np.ones(48), 1e-12)
+    np.testing.assert_allclose(np.sqrt(np.mean(y2.reshape(40, 48) ** 2, axis=1)), 1.0, rtol=1e-9)
