@@ -309,7 +309,6 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         tc_fence_after();
         issue_s(0, 0);
         if (has_q1) issue_s(1, 0);
-        mma_commit(&bars.k_empty[0]);
       }
       for (int i = 0; ok && i < n_tiles; ++i) {
         const uint32_t par = (uint32_t)i & 1u;
@@ -338,11 +337,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
           tc_fence_after();
           issue_pv(1, i);
         }
-        mma_commit(&bars.v_empty[i % C::kVStages]);
-        if (more) {
-          if (has_q1) issue_s(1, i + 1);
-          mma_commit(&bars.k_empty[(i + 1) % C::kKStages]);
-        }
+        if (more && has_q1) issue_s(1, i + 1);
       }
       if (ok) {
         mma_commit(&bars.o_final);
@@ -397,11 +392,22 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
                             p.frame_tokens;
       float m = -INFINITY;  // running max of scale*log2(e)*logit (possibly stale by < threshold)
       float l = 0.0f;       // running sum of 2^(x - m)
+      // The commit that completes the last S of key tile i (S_1, or S_0
+      // without a second query tile) follows every MMA that reads K stage i
+      // and every PV of tile i-1, so one thread of that warpgroup hands K
+      // stage i and V stage i-1 back to the producer as soon as it sees S.
+      // The single MMA-issuing thread then commits only to the two S
+      // barriers per tile (a commit costs it about as long as an MMA issue).
+      const bool releases = b == (has_q1 ? 1 : 0) && q4 == 0 && lane == 0;
       bool ok = true;
       for (int i = 0; i < n_tiles; ++i) {
         ok = mbar_wait(&bars.s_full[b], (uint32_t)i & 1u, &abort_flag, tmo);
         ok = __all_sync(0xffffffffu, ok);
         if (!ok) break;
+        if (releases) {
+          mbar_arrive(&bars.k_empty[i % C::kKStages]);
+          if (i > 0) mbar_arrive(&bars.v_empty[(i - 1) % C::kVStages]);
+        }
         tc_fence_after();
         const int t = (t_begin + i) % p.nt_slot;  // key tile inside its slot
         int valid = (t == p.nt_slot - 1) ? p.valid_last : kTile;
