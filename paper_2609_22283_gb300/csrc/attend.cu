@@ -264,14 +264,16 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+    // The whole warp runs the loop (waits are voted warp-wide so every lane
+    // takes the same branch); one elected lane issues each MMA and commit.
+    {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(128, 128, false);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(128, D, true);
       // Base descriptors are built once; an MMA's operand descriptor is its
       // base plus a compile-time offset (the start-address field holds
       // address >> 4 and every operand lies below 256 KB, so the add never
       // carries out of the field).  Rebuilding descriptors per MMA costs the
-      // single issuing thread about as long as the MMA itself takes.
+      // issuing warp about as long as the MMA itself takes.
       const uint64_t dQ[2] = {sdesc_sw128(smem_u32(sQ0), 16, 1024),
                               sdesc_sw128(smem_u32(sQ1), 16, 1024)};
       const uint64_t dK = sdesc_sw128(smem_u32(sK), 16, 1024);
@@ -285,9 +287,9 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint64_t off = (uint64_t)(((kk >> 2) * C::kBoxBytes + (kk & 3) * 32) >> 4);
-          mma_ss(dcol, qb + off, kb + off, idesc_qk, kk > 0 ? 1u : 0u);
+          mma_ss_warp(dcol, qb + off, kb + off, idesc_qk, kk > 0 ? 1u : 0u);
         }
-        mma_commit(&bars.s_full[b]);
+        mma_commit_warp(&bars.s_full[b]);
       };
       // O_b += P_b V_i with P_b read from TMEM over S_b
       auto issue_pv = [&](int b, int i) {
@@ -297,14 +299,17 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         const uint32_t acc0 = i > 0 ? 1u : 0u;
 #pragma unroll
         for (int kk = 0; kk < kTile / 16; ++kk)
-          mma_ts(ocol, pcol + kk * 8, vb + (uint64_t)((kk * 2048) >> 4), idesc_pv,
+          mma_ts_warp(ocol, pcol + kk * 8, vb + (uint64_t)((kk * 2048) >> 4), idesc_pv,
                  kk > 0 ? 1u : acc0);
       };
-      auto wait_k = [&](int i) {
-        return mbar_wait(&bars.k_full[i % C::kKStages], (uint32_t)(i / C::kKStages) & 1u,
-                         &abort_flag, tmo);
+      auto wait = [&](uint64_t* bar, uint32_t parity) {
+        return __all_sync(0xffffffffu, mbar_wait(bar, parity, &abort_flag, tmo));
       };
-      bool ok = mbar_wait(&bars.q_full, 0, &abort_flag, tmo) && wait_k(0);
+      auto wait_k = [&](int i) {
+        return wait(&bars.k_full[i % C::kKStages], (uint32_t)(i / C::kKStages) & 1u);
+      };
+      bool ok = wait(&bars.q_full, 0);
+      ok = ok && wait_k(0);
       if (ok) {
         tc_fence_after();
         issue_s(0, 0);
@@ -312,9 +317,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       }
       for (int i = 0; ok && i < n_tiles; ++i) {
         const uint32_t par = (uint32_t)i & 1u;
-        if (!mbar_wait(&bars.p_full[0], par, &abort_flag, tmo) ||
-            !mbar_wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u,
-                       &abort_flag, tmo)) {
+        if (!wait(&bars.p_full[0], par) ||
+            !wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u)) {
           ok = false;
           break;
         }
@@ -330,7 +334,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
           issue_s(0, i + 1);
         }
         if (has_q1) {
-          if (!mbar_wait(&bars.p_full[1], par, &abort_flag, tmo)) {
+          if (!wait(&bars.p_full[1], par)) {
             ok = false;
             break;
           }
@@ -340,8 +344,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         if (more && has_q1) issue_s(1, i + 1);
       }
       if (ok) {
-        mma_commit(&bars.o_final);
-      } else {
+        mma_commit_warp(&bars.o_final);
+      } else if (lane == 0) {
         record_timeout(p, &abort_flag);
       }
     }
@@ -350,13 +354,13 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     __syncwarp();
     tc_fence_before();
     __syncthreads();
-    if (abort_flag && lane == 0) {
+    if (abort_flag) {
       // Some wait expired.  Before the CTA exits, wait (bounded, ignoring
       // the abort flag) for what this CTA still has in flight: the TMA
       // copies the producer started (a stage's barrier cannot run ahead of
       // the last copy started into it) and every MMA the issuer started.
       const int zero = 0;
-      if (warp == 0) {
+      if (warp == 0 && lane == 0) {
         mbar_wait(&bars.q_full, 0, &zero, tmo);
         for (int i = (k_issued > C::kKStages ? k_issued - C::kKStages : 0); i < k_issued; ++i)
           mbar_wait(&bars.k_full[i % C::kKStages], (uint32_t)(i / C::kKStages) & 1u, &zero, tmo);
@@ -365,7 +369,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
           mbar_wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u, &zero, tmo);
         }
       } else if (warp == 1) {
-        mma_commit(&bars.drain);
+        mma_commit_warp(&bars.drain);  // the same elected lane that issued the MMAs
         mbar_wait(&bars.drain, 0, &zero, tmo);
       }
     }
@@ -396,8 +400,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       // without a second query tile) follows every MMA that reads K stage i
       // and every PV of tile i-1, so one thread of that warpgroup hands K
       // stage i and V stage i-1 back to the producer as soon as it sees S.
-      // The single MMA-issuing thread then commits only to the two S
-      // barriers per tile (a commit costs it about as long as an MMA issue).
+      // The MMA warp then commits only to the two S barriers per tile (a
+      // commit costs it about as long as an MMA issue).
       const bool releases = b == (has_q1 ? 1 : 0) && q4 == 0 && lane == 0;
       bool ok = true;
       for (int i = 0; i < n_tiles; ++i) {
