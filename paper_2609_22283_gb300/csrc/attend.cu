@@ -317,22 +317,17 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       }
       for (int i = 0; ok && i < n_tiles; ++i) {
         const uint32_t par = (uint32_t)i & 1u;
-        if (!wait(&bars.p_full[0], par) ||
-            !wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u)) {
+        const bool more = i + 1 < n_tiles;
+        // V_i and K_{i+1} land long before the softmax hands over P_0, so
+        // their waits go first, off the path from P_0 to the next MMA.
+        if (!wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u) ||
+            (more && !wait_k(i + 1)) || !wait(&bars.p_full[0], par)) {
           ok = false;
           break;
         }
         tc_fence_after();
         issue_pv(0, i);
-        const bool more = i + 1 < n_tiles;
-        if (more) {
-          if (!wait_k(i + 1)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          issue_s(0, i + 1);
-        }
+        if (more) issue_s(0, i + 1);
         if (has_q1) {
           if (!wait(&bars.p_full[1], par)) {
             ok = false;
@@ -420,33 +415,41 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
           // row's latent frame are visible (tile 0, frame 0, always is)
           valid = min(valid, frame_end - t * kTile);
         }
+        // The loads also reduce each 32-column chunk to its maximum, so a
+        // full tile needs no max tree; a tile with masked keys (the ragged
+        // last tile of a slot, frame causality) takes the max over what is
+        // left after masking.
         uint32_t s[4][32];
+        float cmax[4];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_ld32(scol + c * 32, s[c]);
+        for (int c = 0; c < 4; ++c) tmem_ld32_max(scol + c * 32, s[c], cmax[c]);
 #pragma unroll
         for (int c = 0; c < 4; ++c) tmem_wait_ld(s[c]);
-        if (__any_sync(0xffffffffu, valid < kTile)) {
+        tmem_wait_ld_max(cmax);
+        const bool partial = __any_sync(0xffffffffu, valid < kTile);
+        float m_tile = fmaxf(max3(cmax[0], cmax[1], cmax[2]), cmax[3]) * sl2;
+        if (partial) {
 #pragma unroll
           for (int c = 0; c < 4; ++c)
 #pragma unroll
             for (int e = 0; e < 32; ++e)
               if (c * 32 + e >= valid) s[c][e] = __float_as_uint(-INFINITY);
+          float mx[8];
+#pragma unroll
+          for (int k = 0; k < 8; ++k) mx[k] = -INFINITY;
+#pragma unroll
+          for (int c = 0; c < 4; ++c)
+#pragma unroll
+            for (int e = 0; e < 32; e += 8) {
+              const int k = (c & 1) * 4 + (e >> 3);
+              mx[k] = max3(mx[k], __uint_as_float(s[c][e]), __uint_as_float(s[c][e + 1]));
+              mx[k] = max3(mx[k], __uint_as_float(s[c][e + 2]), __uint_as_float(s[c][e + 3]));
+              mx[k] = max3(mx[k], __uint_as_float(s[c][e + 4]), __uint_as_float(s[c][e + 5]));
+              mx[k] = max3(mx[k], __uint_as_float(s[c][e + 6]), __uint_as_float(s[c][e + 7]));
+            }
+          m_tile =
+              max3(max3(mx[0], mx[1], mx[2]), max3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])) * sl2;
         }
-        float mx[8];
-#pragma unroll
-        for (int k = 0; k < 8; ++k) mx[k] = -INFINITY;
-#pragma unroll
-        for (int c = 0; c < 4; ++c)
-#pragma unroll
-          for (int e = 0; e < 32; e += 8) {
-            const int k = (c & 1) * 4 + (e >> 3);
-            mx[k] = max3(mx[k], __uint_as_float(s[c][e]), __uint_as_float(s[c][e + 1]));
-            mx[k] = max3(mx[k], __uint_as_float(s[c][e + 2]), __uint_as_float(s[c][e + 3]));
-            mx[k] = max3(mx[k], __uint_as_float(s[c][e + 4]), __uint_as_float(s[c][e + 5]));
-            mx[k] = max3(mx[k], __uint_as_float(s[c][e + 6]), __uint_as_float(s[c][e + 7]));
-          }
-        const float m_tile =
-            max3(max3(mx[0], mx[1], mx[2]), max3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])) * sl2;
         const float m_new = fmaxf(m, m_tile);
         const bool need = m_new > m + kRescaleThreshold;
         if (__any_sync(0xffffffffu, need)) {

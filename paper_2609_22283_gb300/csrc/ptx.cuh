@@ -281,9 +281,30 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
 // Waits for this thread's outstanding tensor-memory loads.  Taking the
 // registers as read-write operands keeps the compiler from hoisting their
 // uses above the wait.
+// tmem_ld32 that also returns the maximum of the 32 loaded fp32 values
+// (tcgen05.ld.red, sm_103a): a row max of S without a max tree in registers.
+// `mx`, like the registers, is valid only after a tcgen05.wait::ld that
+// names it (tmem_wait_ld_max).
+__device__ __forceinline__ void tmem_ld32_max(uint32_t taddr, uint32_t (&r)[32], float& mx) {
+  asm volatile(
+      "tcgen05.ld.red.sync.aligned.32x32b.x32.max.f32"
+      " {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, %32, [%33];"
+      : SVA_R8(0), SVA_R8(8), SVA_R8(16), SVA_R8(24), "=f"(mx)
+      : "r"(taddr));
+}
+
 __device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;"
                : SVA_RW8(0), SVA_RW8(8), SVA_RW8(16), SVA_RW8(24)
+               :
+               : "memory");
+}
+
+// Orders reads of four tmem_ld32_max results after the loads completed.
+__device__ __forceinline__ void tmem_wait_ld_max(float (&mx)[4]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;"
+               : "+f"(mx[0]), "+f"(mx[1]), "+f"(mx[2]), "+f"(mx[3])
                :
                : "memory");
 }
