@@ -13,15 +13,17 @@
 // in shared memory serves both query tiles.
 //   warp 0     TMA producer: Q0/Q1 once, then K and V tiles of the slot list
 //              into rings of shared-memory stages (128B swizzle);
-//   warp 1     MMA issuer (one thread) and TMEM owner;
-//   warps 4-7  softmax of Q0, warps 8-11 softmax of Q1: one query row per
-//              thread; S from TMEM, fp32 online softmax in the log2 domain
-//              with a lazy rescale of O, P written back over S as bf16; then
-//              the epilogue (O / l to bf16 global, optional LSE).
+//   warp 1     MMA issuer (the whole warp runs the loop, one elected lane
+//              issues) and TMEM owner;
+//   warps 4-11 softmax, all eight warps on one query tile at a time (Q0 then
+//              Q1 of every key tile): two threads per query row, 64 keys
+//              each; S from TMEM, fp32 online softmax in the log2 domain with
+//              a lazy rescale of O, P written back over S as bf16; then the
+//              epilogue (O / l to bf16 global, optional LSE).
 // TMEM columns: S0 [0,128), S1 [128,256), O0 [256, 256+d), O1 [384, 384+d).
-// MMA order per key tile i: PV0_i, S0_{i+1}, PV1_i, S1_{i+1}, so either
-// softmax warpgroup has the other tile's PV and S (two 128x128x128 MMAs) to
-// hide behind.  A commit that completes S_b of tile i also implies PV_b of
+// MMA order per key tile i: PV0_i, S0_{i+1}, PV1_i, S1_{i+1}, so the softmax
+// of either query tile has the other tile's PV and S (two 128x128x128 MMAs)
+// to hide behind.  A commit that completes S_b of tile i also implies PV_b of
 // tile i-1 is complete (MMAs execute in issue order), so the rescale of O_b
 // needs no extra barrier.
 // A unit may be split into n_split contiguous key ranges (when there are too
@@ -64,11 +66,10 @@ __device__ __forceinline__ uint32_t col_s(int b) { return b ? 128u : 0u; }
 __device__ __forceinline__ uint32_t col_o(int b) { return b ? 384u : 256u; }
 
 // 12 warps: warpgroup 0 = TMA producer (warp 0), MMA issuer (warp 1), two
-// idle warps; warpgroups 1 and 2 = softmax of query tiles 0 and 1.  The
-// launch gives every thread kLaunchRegs registers; warpgroup 0 then gives
-// registers back (setmaxnreg.dec to kRegsLow) and the softmax warpgroups
-// take them (setmaxnreg.inc to kRegsHigh), so a softmax thread can hold a
-// whole 128-key row of S.  The split must fit the launch's pool:
+// idle warps; warpgroups 1 and 2 = softmax.  The launch gives every thread
+// kLaunchRegs registers; warpgroup 0 then gives registers back
+// (setmaxnreg.dec to kRegsLow) and the softmax warpgroups take them
+// (setmaxnreg.inc to kRegsHigh).  The split must fit the launch's pool:
 // 4*32*kRegsLow + 8*32*kRegsHigh <= 384*kLaunchRegs, checked at launch.
 constexpr int kThreads = 384;
 constexpr int kLaunchRegs = 168;
@@ -181,7 +182,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     mbar_init(&bars.drain, 1);
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bars.s_full[b], 1);
-      mbar_init(&bars.p_full[b], 128);
+      mbar_init(&bars.p_full[b], 256);
     }
     for (int s = 0; s < C::kKStages; ++s) {
       mbar_init(&bars.k_full[s], 1);
@@ -376,112 +377,125 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
   } else {
     regs_inc<kRegsHigh>();
     // ------------------------------------------------------------ softmax + epilogue
-    const int b = (warp >> 2) - 1;                 // query tile of this warpgroup
+    // All eight softmax warps work on one query tile at a time (tile 0, then
+    // tile 1, of every key tile).  A warp covers 16 rows, half of its TMEM
+    // lane quarter, with two threads per row (16x32bx2 shape): thread t < 16
+    // holds keys 0..63 of its row, thread t + 16 keys 64..127 of the same
+    // row.  Both threads of a row keep the same running max (the two halves'
+    // maxima are exchanged with one shuffle) and each its part of the sum,
+    // so each thread exponentiates 64 keys per tile instead of 128 and the
+    // two warps sharing a sub-partition overlap their MUFU and FMA work.
+    constexpr int DH = D / 2;                      // output columns per thread
     const int q4 = warp & 3;                       // TMEM lane quarter this warp may access
-    const int row = q4 * 32 + lane;                // query row inside the tile
-    const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
-    if (b == 0 || has_q1) {
-      const float sl2 = p.scale_log2;
-      const uint64_t sl2x2 = f2u(sl2, sl2);
-      const uint32_t scol = tbase + lane_off + col_s(b);
-      const uint32_t ocol = tbase + lane_off + col_o(b);
-      const int frame_causal = nd.frame_causal;
-      // first token of the latent frame after this row's (frame-causal mask)
-      const int frame_end = ((qt0 + b) * kTile + row) / p.frame_tokens * p.frame_tokens +
-                            p.frame_tokens;
-      float m = -INFINITY;  // running max of scale*log2(e)*logit (possibly stale by < threshold)
-      float l = 0.0f;       // running sum of 2^(x - m)
-      // The commit that completes the last S of key tile i (S_1, or S_0
-      // without a second query tile) follows every MMA that reads K stage i
-      // and every PV of tile i-1, so one thread of that warpgroup hands K
-      // stage i and V stage i-1 back to the producer as soon as it sees S.
-      // The MMA warp then commits only to the two S barriers per tile (a
-      // commit costs it about as long as an MMA issue).
-      const bool releases = b == (has_q1 ? 1 : 0) && q4 == 0 && lane == 0;
-      bool ok = true;
-      for (int i = 0; i < n_tiles; ++i) {
+    const int hi = warp >> 3;                      // which 16 lanes of the quarter
+    const int half = lane >> 4;                    // which 64 keys, which D/2 columns
+    const int row = q4 * 32 + hi * 16 + (lane & 15);  // query row inside a tile
+    const uint32_t lane_off = (uint32_t)(q4 * 32 + hi * 16) << 16;
+    const int nb = has_q1 ? 2 : 1;
+    const float sl2 = p.scale_log2;
+    const uint64_t sl2x2 = f2u(sl2, sl2);
+    const int frame_causal = nd.frame_causal;
+    float m[2] = {-INFINITY, -INFINITY};  // running max of scale*log2(e)*logit per query tile
+    float l[2] = {0.0f, 0.0f};            // this thread's part of the running sum of 2^(x - m)
+    // first token of the latent frame after this row's (frame-causal mask)
+    int frame_end[2];
+#pragma unroll
+    for (int b = 0; b < 2; ++b)
+      frame_end[b] = ((qt0 + b) * kTile + row) / p.frame_tokens * p.frame_tokens + p.frame_tokens;
+    // The commit that completes the last S of key tile i (S_1, or S_0
+    // without a second query tile) follows every MMA that reads K stage i
+    // and every PV of tile i-1, so one softmax thread hands K stage i and V
+    // stage i-1 back to the producer as soon as it sees that S.  The MMA
+    // warp then commits only to the two S barriers per tile (a commit costs
+    // it about as long as an MMA issue).
+    const bool releaser = warp == 4 && lane == 0;
+    bool ok = true;
+    for (int i = 0; ok && i < n_tiles; ++i) {
+      const int t = (t_begin + i) % p.nt_slot;  // key tile inside its slot
+      const int valid_tile = (t == p.nt_slot - 1) ? p.valid_last : kTile;
+      const bool own_fc = frame_causal && t_begin + i < p.nt_slot;
+#pragma unroll
+      for (int b = 0; b < 2; ++b) {
+        if (b == 1 && !has_q1) break;
         ok = mbar_wait(&bars.s_full[b], (uint32_t)i & 1u, &abort_flag, tmo);
         ok = __all_sync(0xffffffffu, ok);
         if (!ok) break;
-        if (releases) {
+        if (releaser && b == nb - 1) {
           mbar_arrive(&bars.k_empty[i % C::kKStages]);
           if (i > 0) mbar_arrive(&bars.v_empty[(i - 1) % C::kVStages]);
         }
         tc_fence_after();
-        const int t = (t_begin + i) % p.nt_slot;  // key tile inside its slot
-        int valid = (t == p.nt_slot - 1) ? p.valid_last : kTile;
-        if (frame_causal && t_begin + i < p.nt_slot) {
-          // own-chunk tile under frame causality: keys up to the end of this
-          // row's latent frame are visible (tile 0, frame 0, always is)
-          valid = min(valid, frame_end - t * kTile);
-        }
+        const uint32_t scol = tbase + lane_off + col_s(b);
+        const uint32_t ocol = tbase + lane_off + col_o(b);
+        // own-chunk tile under frame causality: keys up to the end of this
+        // row's latent frame are visible (tile 0, frame 0, always is)
+        const int valid = own_fc ? min(valid_tile, frame_end[b] - t * kTile) : valid_tile;
+        const int vrel = valid - half * 64;  // visible keys among this thread's 64
         // The loads also reduce each 32-column chunk to its maximum, so a
         // full tile needs no max tree; a tile with masked keys (the ragged
         // last tile of a slot, frame causality) takes the max over what is
         // left after masking.
-        uint32_t s[4][32];
-        float cmax[4];
+        uint32_t s[2][32];
+        float cmax[2];
+        tmem_ld16x2_32_max<64>(scol, s[0], cmax[0]);
+        tmem_ld16x2_32_max<64>(scol + 32, s[1], cmax[1]);
+        tmem_wait_ld(s[0]);
+        tmem_wait_ld(s[1]);
+        tmem_wait_ld_max2(cmax);
+        float m_part = fmaxf(cmax[0], cmax[1]);
+        if (__any_sync(0xffffffffu, vrel < 64)) {
+          float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_ld32_max(scol + c * 32, s[c], cmax[c]);
-#pragma unroll
-        for (int c = 0; c < 4; ++c) tmem_wait_ld(s[c]);
-        tmem_wait_ld_max(cmax);
-        const bool partial = __any_sync(0xffffffffu, valid < kTile);
-        float m_tile = fmaxf(max3(cmax[0], cmax[1], cmax[2]), cmax[3]) * sl2;
-        if (partial) {
-#pragma unroll
-          for (int c = 0; c < 4; ++c)
+          for (int c = 0; c < 2; ++c)
 #pragma unroll
             for (int e = 0; e < 32; ++e)
-              if (c * 32 + e >= valid) s[c][e] = __float_as_uint(-INFINITY);
-          float mx[8];
+              if (c * 32 + e >= vrel) s[c][e] = __float_as_uint(-INFINITY);
 #pragma unroll
-          for (int k = 0; k < 8; ++k) mx[k] = -INFINITY;
-#pragma unroll
-          for (int c = 0; c < 4; ++c)
+          for (int c = 0; c < 2; ++c)
 #pragma unroll
             for (int e = 0; e < 32; e += 8) {
-              const int k = (c & 1) * 4 + (e >> 3);
+              const int k = (c & 1) * 2 + (e >> 4);
               mx[k] = max3(mx[k], __uint_as_float(s[c][e]), __uint_as_float(s[c][e + 1]));
               mx[k] = max3(mx[k], __uint_as_float(s[c][e + 2]), __uint_as_float(s[c][e + 3]));
               mx[k] = max3(mx[k], __uint_as_float(s[c][e + 4]), __uint_as_float(s[c][e + 5]));
               mx[k] = max3(mx[k], __uint_as_float(s[c][e + 6]), __uint_as_float(s[c][e + 7]));
             }
-          m_tile =
-              max3(max3(mx[0], mx[1], mx[2]), max3(mx[3], mx[4], mx[5]), fmaxf(mx[6], mx[7])) * sl2;
+          m_part = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3]));
         }
-        const float m_new = fmaxf(m, m_tile);
-        const bool need = m_new > m + kRescaleThreshold;
+        const float m_tile = fmaxf(m_part, __shfl_xor_sync(0xffffffffu, m_part, 16)) * sl2;
+        const float m_new = fmaxf(m[b], m_tile);
+        const bool need = m_new > m[b] + kRescaleThreshold;
         if (__any_sync(0xffffffffu, need)) {
-          const float alpha = ex2(m - m_new);  // 0 on the first tile (m = -inf)
+          const float alpha = ex2(m[b] - m_new);  // 0 on the first tile (m = -inf)
           if (i > 0) {
             // O_b holds the sum over tiles < i: the commit that completed S_b
             // of tile i came after PV_b of tile i-1.
 #pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
+            for (int c = 0; c < DH / 32; ++c) {
               uint32_t o[32];
-              tmem_ld32(ocol + c * 32, o);
+              tmem_ld16x2_32<DH>(ocol + c * 32, o);
               tmem_wait_ld(o);
 #pragma unroll
               for (int e = 0; e < 32; ++e) o[e] = __float_as_uint(__uint_as_float(o[e]) * alpha);
-              tmem_st32(ocol + c * 32, o);
+              tmem_st16x2_32<DH>(ocol + c * 32, o);
             }
             tmem_wait_st();
           }
-          l *= alpha;
-          m = m_new;
+          l[b] *= alpha;
+          m[b] = m_new;
         }
         // m stays -inf while a row has seen no visible key (possible in a key
         // range that starts past a row's frame under frame causality); its
         // scores are then all -inf and must give P = 0, not NaN.
-        const float m_sub = (m == -INFINITY) ? 0.0f : m;
+        const float m_sub = (m[b] == -INFINITY) ? 0.0f : m[b];
         const uint64_t negm = f2u(-m_sub, -m_sub);
         uint64_t acc[4] = {0, 0, 0, 0};
         // P of 32 keys packs into 16 words, written over the first half of
         // the same registers (word e/2 is written after elements e, e+1 are
-        // read); two such halves make one 32-column store over S.
+        // read); the two halves make one 32-column store over S (keys
+        // 0..63 of the row at columns 0..31, keys 64..127 at 32..63).
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
+        for (int c = 0; c < 2; ++c) {
 #pragma unroll
           for (int e = 0; e < 32; e += 2) {
             float x0, x1;
@@ -491,36 +505,42 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
             acc[(e >> 1) & 3] = fadd2(acc[(e >> 1) & 3], p0, p1);
             s[c][e >> 1] = pack_bf16(p0, p1);
           }
-          if (c & 1) tmem_st32_halves(scol + (c >> 1) * 32, s[c - 1], s[c]);
         }
+        tmem_st16x2_32_halves<32>(scol, s[0], s[1]);
         float a0, a1, a2, a3, a4, a5, a6, a7;
         u2f(acc[0], a0, a1);
         u2f(acc[1], a2, a3);
         u2f(acc[2], a4, a5);
         u2f(acc[3], a6, a7);
-        l += ((a0 + a1) + (a2 + a3)) + ((a4 + a5) + (a6 + a7));
+        l[b] += ((a0 + a1) + (a2 + a3)) + ((a4 + a5) + (a6 + a7));
         tmem_wait_st();
         tc_fence_before();
         mbar_arrive(&bars.p_full[b]);
       }
-      if (ok) {
-        ok = mbar_wait(&bars.o_final, 0, &abort_flag, tmo);
-        ok = __all_sync(0xffffffffu, ok);
-      }
-      if (!ok) record_timeout(p, &abort_flag);
-      const int token = (qt0 + b) * kTile + row;
-      const bool in_range = token < p.T;
-      __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(p.out) +
-                            (((size_t)nd.q_index * p.T + token) * p.H + h) * D;
-      float* lse_at = p.lse ? p.lse + ((size_t)nd.q_index * p.H + h) * p.T + token : nullptr;
-      if (p.n_split == 1) {
-        if (ok) {
-          tc_fence_after();
-          const float inv_l = l > 0.0f ? 1.0f / l : 0.0f;  // a row with no visible key: O = 0
+    }
+    if (ok) {
+      ok = mbar_wait(&bars.o_final, 0, &abort_flag, tmo);
+      ok = __all_sync(0xffffffffu, ok);
+    }
+    if (!ok) record_timeout(p, &abort_flag);
+    float l_row[2];  // the row's whole sum: both halves, under the same max
 #pragma unroll
-          for (int c = 0; c < D / 32; ++c) {
+    for (int b = 0; b < 2; ++b) l_row[b] = l[b] + __shfl_xor_sync(0xffffffffu, l[b], 16);
+    if (p.n_split == 1) {
+      if (ok) {
+        tc_fence_after();
+#pragma unroll
+        for (int b = 0; b < 2; ++b) {
+          if (b == 1 && !has_q1) break;
+          const int token = (qt0 + b) * kTile + row;
+          const bool in_range = token < p.T;
+          __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(p.out) +
+                                (((size_t)nd.q_index * p.T + token) * p.H + h) * D + DH * half;
+          const float inv_l = l_row[b] > 0.0f ? 1.0f / l_row[b] : 0.0f;  // no visible key: O = 0
+#pragma unroll
+          for (int c = 0; c < DH / 32; ++c) {
             uint32_t o[32];
-            tmem_ld32(ocol + c * 32, o);
+            tmem_ld16x2_32<DH>(tbase + lane_off + col_o(b) + c * 32, o);
             tmem_wait_ld(o);
             if (in_range) {
               uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
@@ -535,46 +555,60 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
               }
             }
           }
-          if (lse_at != nullptr && in_range) *lse_at = (m + __log2f(l)) * 0.69314718055994531f;
+          if (p.lse != nullptr && in_range && half == 0)
+            p.lse[((size_t)nd.q_index * p.H + h) * p.T + token] =
+                (m[b] + __log2f(l_row[b])) * 0.69314718055994531f;
         }
-      } else {
-        // Split unit.  Partial layout per (unit, split): O as [D/4][256]
-        // float4 (rows of both query tiles), then m[256], then l[256].
-        constexpr size_t kItem = (size_t)256 * (D + 2);
-        const int r = b * 128 + row;
-        float* part = p.ws + ((size_t)unit * p.n_split + split) * kItem;
-        if (ok) {
-          tc_fence_after();
-          const float inv_l = l > 0.0f ? 1.0f / l : 0.0f;  // no visible key in this range
-          float4* part4 = reinterpret_cast<float4*>(part);
+      }
+    } else {
+      // Split unit.  Partial layout per (unit, split): O as [D/4][256]
+      // float4 (rows of both query tiles), then m[256], then l[256].
+      constexpr size_t kItem = (size_t)256 * (D + 2);
+      float* part = p.ws + ((size_t)unit * p.n_split + split) * kItem;
+      if (ok) {
+        tc_fence_after();
+        float4* part4 = reinterpret_cast<float4*>(part);
 #pragma unroll
-          for (int c = 0; c < D / 32; ++c) {
+        for (int b = 0; b < 2; ++b) {
+          if (b == 1 && !has_q1) break;
+          const int r = b * 128 + row;
+          const float inv_l = l_row[b] > 0.0f ? 1.0f / l_row[b] : 0.0f;  // no visible key here
+#pragma unroll
+          for (int c = 0; c < DH / 32; ++c) {
             uint32_t o[32];
-            tmem_ld32(ocol + c * 32, o);
+            tmem_ld16x2_32<DH>(tbase + lane_off + col_o(b) + c * 32, o);
             tmem_wait_ld(o);
 #pragma unroll
             for (int v = 0; v < 8; ++v)
-              part4[(c * 8 + v) * 256 + r] =
+              part4[(DH * half / 4 + c * 8 + v) * 256 + r] =
                   make_float4(__uint_as_float(o[v * 4 + 0]) * inv_l, __uint_as_float(o[v * 4 + 1]) * inv_l,
                               __uint_as_float(o[v * 4 + 2]) * inv_l, __uint_as_float(o[v * 4 + 3]) * inv_l);
           }
-          part[D * 256 + r] = m;
-          part[D * 256 + 256 + r] = l;
+          if (half == 0) {
+            part[D * 256 + r] = m[b];
+            part[D * 256 + 256 + r] = l_row[b];
+          }
         }
+      }
+      __threadfence();
+      // Every softmax thread of the CTA passes both barriers, whatever its
+      // wait results were, so none can be left waiting here.
+      asm volatile("bar.sync 1, 256;" ::: "memory");
+      if (threadIdx.x == 128) {
+        int last = 0;
+        if (!abort_flag) last = atomicAdd(&p.ws_count[unit], 1) == p.n_split - 1;
+        last_split = last;
+      }
+      asm volatile("bar.sync 1, 256;" ::: "memory");
+      if (last_split) {
         __threadfence();
-        // Every softmax thread of the CTA passes both barriers, whatever its
-        // wait results were, so none can be left waiting here.
-        const uint32_t nsoft = has_q1 ? 256u : 128u;
-        asm volatile("bar.sync 1, %0;" ::"r"(nsoft) : "memory");
-        if (threadIdx.x == 128) {
-          int last = 0;
-          if (!abort_flag) last = atomicAdd(&p.ws_count[unit], 1) == p.n_split - 1;
-          last_split = last;
-        }
-        asm volatile("bar.sync 1, %0;" ::"r"(nsoft) : "memory");
-        if (last_split) {
-          __threadfence();
-          const float* base = p.ws + (size_t)unit * p.n_split * kItem;
+        const float* base = p.ws + (size_t)unit * p.n_split * kItem;
+#pragma unroll
+        for (int b = 0; b < 2; ++b) {
+          if (b == 1 && !has_q1) break;
+          const int r = b * 128 + row;
+          const int token = (qt0 + b) * kTile + row;
+          if (token >= p.T) continue;
           float mk[kMaxSplit], wk[kMaxSplit];
           float M = -INFINITY;
 #pragma unroll
@@ -594,30 +628,31 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
           const float inv_L = L > 0.0f ? 1.0f / L : 0.0f;
 #pragma unroll
           for (int k = 0; k < kMaxSplit; ++k) wk[k] *= inv_L;
-          if (in_range) {
+          uint4* orow4 = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(p.out) +
+                                                  (((size_t)nd.q_index * p.T + token) * p.H + h) * D);
 #pragma unroll 4
-            for (int c8 = 0; c8 < D / 8; ++c8) {
-              float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+          for (int c8 = half * (D / 16); c8 < (half + 1) * (D / 16); ++c8) {
+            float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-              for (int k = 0; k < kMaxSplit; ++k) {
-                if (k >= p.n_split) break;
-                const float4* b4 = reinterpret_cast<const float4*>(base + k * kItem);
-                const float4 x = __ldcg(b4 + (c8 * 2 + 0) * 256 + r);
-                const float4 y = __ldcg(b4 + (c8 * 2 + 1) * 256 + r);
-                a[0] += wk[k] * x.x; a[1] += wk[k] * x.y; a[2] += wk[k] * x.z; a[3] += wk[k] * x.w;
-                a[4] += wk[k] * y.x; a[5] += wk[k] * y.y; a[6] += wk[k] * y.z; a[7] += wk[k] * y.w;
-              }
-              uint4 w;
-              w.x = pack_bf16(a[0], a[1]);
-              w.y = pack_bf16(a[2], a[3]);
-              w.z = pack_bf16(a[4], a[5]);
-              w.w = pack_bf16(a[6], a[7]);
-              reinterpret_cast<uint4*>(orow)[c8] = w;
+            for (int k = 0; k < kMaxSplit; ++k) {
+              if (k >= p.n_split) break;
+              const float4* b4 = reinterpret_cast<const float4*>(base + k * kItem);
+              const float4 x = __ldcg(b4 + (c8 * 2 + 0) * 256 + r);
+              const float4 y = __ldcg(b4 + (c8 * 2 + 1) * 256 + r);
+              a[0] += wk[k] * x.x; a[1] += wk[k] * x.y; a[2] += wk[k] * x.z; a[3] += wk[k] * x.w;
+              a[4] += wk[k] * y.x; a[5] += wk[k] * y.y; a[6] += wk[k] * y.z; a[7] += wk[k] * y.w;
             }
-            if (lse_at != nullptr) *lse_at = (M + __log2f(L)) * 0.69314718055994531f;
+            uint4 w;
+            w.x = pack_bf16(a[0], a[1]);
+            w.y = pack_bf16(a[2], a[3]);
+            w.z = pack_bf16(a[4], a[5]);
+            w.w = pack_bf16(a[6], a[7]);
+            orow4[c8] = w;
           }
-          if (threadIdx.x == 128) p.ws_count[unit] = 0;  // ready for the next launch
+          if (p.lse != nullptr && half == 0)
+            p.lse[((size_t)nd.q_index * p.H + h) * p.T + token] = (M + __log2f(L)) * 0.69314718055994531f;
         }
+        if (threadIdx.x == 128) p.ws_count[unit] = 0;  // ready for the next launch
       }
     }
     // ---------------------------------------------------------------- teardown (softmax)

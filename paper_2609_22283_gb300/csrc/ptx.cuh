@@ -301,6 +301,63 @@ __device__ __forceinline__ void tmem_wait_ld(uint32_t (&r)[32]) {
                : "memory");
 }
 
+// 16-lane forms (shape 16x32bx2): a warp reads or writes 16 TMEM lanes (its
+// lane quarter's half at the address), and the two half-warps take different
+// columns: thread t < 16 gets lane t at columns [c, c + 32), thread t >= 16
+// gets lane t - 16 at columns [c + OFF, c + OFF + 32).  So two threads share
+// one row and each holds 32 consecutive columns of it.
+template <int OFF>
+__device__ __forceinline__ void tmem_ld16x2_32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.16x32bx2.x32.b32"
+      " {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32], %33;"
+      : SVA_R8(0), SVA_R8(8), SVA_R8(16), SVA_R8(24)
+      : "r"(taddr), "n"(OFF));
+}
+
+// tmem_ld16x2_32 that also returns the maximum of the thread's 32 values.
+template <int OFF>
+__device__ __forceinline__ void tmem_ld16x2_32_max(uint32_t taddr, uint32_t (&r)[32], float& mx) {
+  asm volatile(
+      "tcgen05.ld.red.sync.aligned.16x32bx2.x32.max.f32"
+      " {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, %32, [%33], %34;"
+      : SVA_R8(0), SVA_R8(8), SVA_R8(16), SVA_R8(24), "=f"(mx)
+      : "r"(taddr), "n"(OFF));
+}
+
+template <int OFF>
+__device__ __forceinline__ void tmem_st16x2_32(uint32_t taddr, const uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.16x32bx2.x32.b32 [%0], %33,"
+      " {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      SVA_W8(0), SVA_W8(8), SVA_W8(16), SVA_W8(24), "n"(OFF)
+      : "memory");
+}
+
+// Same as tmem_st16x2_32 with the 32 columns taken from two 16-register halves.
+template <int OFF>
+__device__ __forceinline__ void tmem_st16x2_32_halves(uint32_t taddr, const uint32_t* a,
+                                                      const uint32_t* b) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.16x32bx2.x32.b32 [%0], %33,"
+      " {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16,"
+      "%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(a[4]), "r"(a[5]), "r"(a[6]), "r"(a[7]),
+      "r"(a[8]), "r"(a[9]), "r"(a[10]), "r"(a[11]), "r"(a[12]), "r"(a[13]), "r"(a[14]),
+      "r"(a[15]), "r"(b[0]), "r"(b[1]), "r"(b[2]), "r"(b[3]), "r"(b[4]), "r"(b[5]), "r"(b[6]),
+      "r"(b[7]), "r"(b[8]), "r"(b[9]), "r"(b[10]), "r"(b[11]), "r"(b[12]), "r"(b[13]),
+      "r"(b[14]), "r"(b[15]), "n"(OFF)
+      : "memory");
+}
+
+// Orders reads of tmem_ld*_max results after the loads completed.
+__device__ __forceinline__ void tmem_wait_ld_max2(float (&mx)[2]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" : "+f"(mx[0]), "+f"(mx[1]) : : "memory");
+}
+
 // Orders reads of four tmem_ld32_max results after the loads completed.
 __device__ __forceinline__ void tmem_wait_ld_max(float (&mx)[4]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;"
