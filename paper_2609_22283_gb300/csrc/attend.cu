@@ -630,17 +630,23 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
           for (int k = 0; k < kMaxSplit; ++k) wk[k] *= inv_L;
           uint4* orow4 = reinterpret_cast<uint4*>(static_cast<__nv_bfloat16*>(p.out) +
                                                   (((size_t)nd.q_index * p.T + token) * p.H + h) * D);
-#pragma unroll 4
+          // Loads of absent splits are predicated off rather than broken out
+          // of, so every load of an iteration is in flight at once (a loop
+          // that waited for each L2 round trip in turn took ~9 us per CTA).
+#pragma unroll 2
           for (int c8 = half * (D / 16); c8 < (half + 1) * (D / 16); ++c8) {
+            float4 x[kMaxSplit], y[kMaxSplit];
+#pragma unroll
+            for (int k = 0; k < kMaxSplit; ++k) {
+              const float4* b4 = reinterpret_cast<const float4*>(base + k * kItem);
+              x[k] = k < p.n_split ? __ldcg(b4 + (c8 * 2 + 0) * 256 + r) : make_float4(0.f, 0.f, 0.f, 0.f);
+              y[k] = k < p.n_split ? __ldcg(b4 + (c8 * 2 + 1) * 256 + r) : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
             float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int k = 0; k < kMaxSplit; ++k) {
-              if (k >= p.n_split) break;
-              const float4* b4 = reinterpret_cast<const float4*>(base + k * kItem);
-              const float4 x = __ldcg(b4 + (c8 * 2 + 0) * 256 + r);
-              const float4 y = __ldcg(b4 + (c8 * 2 + 1) * 256 + r);
-              a[0] += wk[k] * x.x; a[1] += wk[k] * x.y; a[2] += wk[k] * x.z; a[3] += wk[k] * x.w;
-              a[4] += wk[k] * y.x; a[5] += wk[k] * y.y; a[6] += wk[k] * y.z; a[7] += wk[k] * y.w;
+              a[0] += wk[k] * x[k].x; a[1] += wk[k] * x[k].y; a[2] += wk[k] * x[k].z; a[3] += wk[k] * x[k].w;
+              a[4] += wk[k] * y[k].x; a[5] += wk[k] * y[k].y; a[6] += wk[k] * y[k].z; a[7] += wk[k] * y[k].w;
             }
             uint4 w;
             w.x = pack_bf16(a[0], a[1]);
