@@ -197,7 +197,7 @@ def attend_rows(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float,
 def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
                  states: dict, q_raw: np.ndarray, heads, rows, scale: float,
                  hidden: frozenset = frozenset(), within: str = "bidirectional",
-                 norm=None):
+                 norm=None, tile_mask=None):
     """One denoising node (seq, b, j), computed from raw (pre-RoPE) inputs.
 
     states: {(seq, chunk, level): (K_raw, V_raw)} with arrays [T][H][d] holding
@@ -211,6 +211,11 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
         frames <= f only); the token-level mask of Eq. 4 either way.
     norm: None, or (gamma_k, gamma_q, eps): every key state's K and the
         node's Q are RMS-normalised per token (rms_norm) before the rotation.
+    tile_mask: None, or a boolean array [query tile][key tile] for the node
+        (query-dependent block-sparse access, Eq. 4 at 128-token tiles):
+        query u (tile u // 128) sees key v of key state s (0 = own chunk,
+        1 + j = j-th selected state) only if entry [u // 128][s * nt + v // 128]
+        is true, nt = ceil(T / 128); a further mask on top of the others.
 
     Steps (Section 3.2): select the context states of the node with Eq. 2-3;
     rotate the K of the node's own state and of every selected state and the
@@ -230,13 +235,21 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
     lse = np.empty((len(heads), len(rows)))
     frame_tokens = g.Hp * g.Wp
     key_frame = np.arange(g.T) // frame_tokens            # latent frame of own-chunk key v
-    # query rows grouped by the mask they get: one group unless frame-causal
-    if within == "frame_causal":
-        groups = [(f, np.nonzero(rows // frame_tokens == f)[0]) for f in range(g.F)]
-    elif within == "bidirectional":
-        groups = [(None, np.arange(len(rows)))]
-    else:
+    key_tile = np.arange(g.T) // 128                     # tile of key v inside its state
+    nt = -(-g.T // 128)
+    if within not in ("frame_causal", "bidirectional"):
         raise ValueError(within)
+    # query rows grouped by the mask they get: by latent frame when
+    # frame-causal, by query tile under a tile mask
+    row_frame = rows // frame_tokens if within == "frame_causal" else np.zeros_like(rows)
+    row_tile = rows // 128 if tile_mask is not None else np.zeros_like(rows)
+    groups = []
+    for f in np.unique(row_frame):
+        for qt in np.unique(row_tile):
+            idx = np.nonzero((row_frame == f) & (row_tile == qt))[0]
+            if len(idx):
+                groups.append((f if within == "frame_causal" else None,
+                               qt if tile_mask is not None else None, idx))
     if norm is not None:
         gk, gq, eps = norm
         states = {s: (rms_norm(states[s][0], gk, eps), states[s][1])
@@ -253,12 +266,14 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
         k = np.concatenate(ks)
         v = np.concatenate(vs)
         q = bf16(rope_head(np.asarray(q_raw[:, h, :], dtype=np.float64), b, g))[rows]
-        for f, idx in groups:
-            if len(idx) == 0:
-                continue
+        for f, qt, idx in groups:
             m = np.concatenate(ms)
             if f is not None:
                 m[:g.T] = np.where(key_frame > f, -np.inf, m[:g.T])   # own chunk comes first
+            if qt is not None:
+                for si in range(len(key_states)):
+                    kept = np.asarray(tile_mask[qt][si * nt + key_tile], dtype=bool)
+                    m[si * g.T:(si + 1) * g.T] = np.where(kept, m[si * g.T:(si + 1) * g.T], -np.inf)
             o, l = attend_rows(q[idx], k, v, scale, m)
             out[hi, idx] = o
             lse[hi, idx] = l

@@ -71,7 +71,8 @@ def _rope(x: np.ndarray, chunk: int, F: int, Hp: int, Wp: int, pairs, theta: flo
 
 def brute_forward(policy: str, W: int, F: int, Hp: int, Wp: int, pairs, theta: float,
                   node: tuple[int, int, int], grid: dict, q_raw: np.ndarray,
-                  heads, scale: float, hidden=frozenset(), frame_causal: bool = False):
+                  heads, scale: float, hidden=frozenset(), frame_causal: bool = False,
+                  tile_mask=None):
     """All query rows of `heads` for node (seq, b, j) against the whole grid.
 
     grid: {(seq, chunk, level): (K_raw, V_raw)} [T][H][d]; it may hold states
@@ -79,6 +80,9 @@ def brute_forward(policy: str, W: int, F: int, Hp: int, Wp: int, pairs, theta: f
     hidden: states whose visibility bit is 0 although the policy selects them.
     frame_causal: inside the own chunk, query token u sees key token v only if
     v's latent frame is not after u's.
+    tile_mask: None, or booleans [query tile][key tile]: query u sees key
+    token v of state (c, l) only if entry [u // 128][r * nt + v // 128] is
+    set, r = b - c (the offset of Eq. 2; 0 for the own chunk), nt = ceil(T/128).
     Returns (out [len(heads)][T][d], lse [len(heads)][T]).
     """
     seq, b, j = node
@@ -101,6 +105,7 @@ def brute_forward(policy: str, W: int, F: int, Hp: int, Wp: int, pairs, theta: f
         M = np.concatenate(mm)
         Q = _bf16_vec(_rope(np.asarray(q_raw[:, h, :], np.float64), b, F, Hp, Wp, pairs, theta))
         own_start = keys.index((seq, b, j)) * T       # where the own chunk sits in the sequence
+        nt = -(-T // 128)
         out = np.zeros((T, d))
         lse = np.zeros(T)
         for u in range(T):
@@ -109,6 +114,13 @@ def brute_forward(policy: str, W: int, F: int, Hp: int, Wp: int, pairs, theta: f
                 for v in range(T):
                     if v // (Hp * Wp) > u // (Hp * Wp):
                         Mu[own_start + v] = -np.inf
+            if tile_mask is not None:
+                for ki, (s, c, l) in enumerate(keys):
+                    if s != seq or not (0 <= b - c) or (b - c) * nt >= len(tile_mask[0]):
+                        continue   # other sequences, future and far chunks: masked anyway
+                    for v in range(T):
+                        if not tile_mask[u // 128][(b - c) * nt + v // 128]:
+                            Mu[ki * T + v] = -np.inf
             logits = [scale * float(np.dot(Q[u], K[v])) + Mu[v] for v in range(K.shape[0])]
             mx = max(logits)
             w = [math.exp(x - mx) if x != -math.inf else 0.0 for x in logits]

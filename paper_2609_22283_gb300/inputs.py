@@ -14,6 +14,9 @@ to bf16, in this order: for each prefilled state (in the listed order) its K
 then its V [T][H][d]; then Q, K_new and V_new [n_nodes][T][H][d].  With
 `outliers`, each draw is followed by a U(0, 1) draw of the same shape on the
 same generator and elements whose uniform is below 0.01 are multiplied by 10.
+
+Block-sparse workloads (`sparse` = a density) also get a seeded key-tile mask
+per (node, query tile), see `tile_mask`.
 """
 from __future__ import annotations
 
@@ -48,6 +51,7 @@ class Workload:
     round: int | None = None  # pipeline round the nodes form (Eq. 6), if any
     within: str = "bidirectional"  # visibility inside the own chunk (or "frame_causal")
     qknorm: bool = False  # RMS-normalise K and Q per token before RoPE (seeded gammas)
+    sparse: float | None = None  # density of kept context key tiles (block-sparse mask), or None
     description: str = ""
     theta: float = 10000.0
     pairs: tuple = field(default=None)
@@ -68,6 +72,17 @@ class Workload:
     def states(self) -> tuple:
         """Every state the step touches: prefilled ones, then the nodes' own."""
         return tuple(self.prefilled) + tuple(self.nodes)
+
+    @property
+    def tiles(self) -> int:
+        """128-token tiles per chunk (query tiles of a node, key tiles of a state)."""
+        return -(-self.T // 128)
+
+    @property
+    def mask_words(self) -> int:
+        """32-bit words per (node, query tile) row of `tile_mask`: room for the own
+        state and up to W context states."""
+        return -(-(1 + self.W) * self.tiles // 32)
 
     @property
     def max_frames(self) -> int:
@@ -128,6 +143,16 @@ WORKLOADS = {
         name="tinyn", seed=10, F=1, Hp=8, Wp=8, H=2, d=64, K=2, W=2, policy="prog",
         nodes=((0, 3, 2), (0, 2, 1)), prefilled=((0, 1, 0),), B=3, round=3, qknorm=True,
         description="tiny with K and Q RMS-normalised per token before RoPE"),
+    "tinys": Workload(
+        name="tinys", seed=11, F=1, Hp=16, Wp=20, H=2, d=64, K=2, W=2, policy="prog",
+        nodes=((0, 3, 2), (0, 2, 1)), prefilled=((0, 1, 0),), B=3, round=3, sparse=0.5,
+        description="tiny with 320-token chunks (3 key tiles, the last 64 rows) and a seeded "
+                    "block-sparse mask keeping half of the context key tiles per query tile"),
+    "prog4s": Workload(
+        name="prog4s", seed=9, F=3, Hp=30, Wp=52, H=12, d=128, K=4, W=6, policy="prog",
+        nodes=_round_nodes(0, 4, 20), prefilled=_PROG_PREFILL_20, round=20, sparse=0.5,
+        description="prog4 with query-dependent block-sparse access: every query tile keeps its "
+                    "own chunk and a seeded half of the 128-token key tiles of its history"),
     "prog4fc": Workload(
         name="prog4fc", seed=8, F=3, Hp=30, Wp=52, H=12, d=128, K=4, W=6, policy="prog",
         nodes=_round_nodes(0, 4, 20), prefilled=_PROG_PREFILL_20, round=20,
@@ -146,7 +171,7 @@ WORKLOADS = {
 # The order the workloads are listed in the configuration table; prog4r adds
 # the clean-state refresh node to prog4's round.
 ORDER = ("tiny", "clean1", "same4", "prog4", "stress14b")
-EXTRA = ("prog4r", "clean5", "tinyfc", "prog4fc", "tinyn")
+EXTRA = ("prog4r", "clean5", "tinyfc", "prog4fc", "tinyn", "tinys", "prog4s")
 
 
 @dataclass
@@ -185,6 +210,45 @@ def generate(w: Workload) -> Inputs:
         inp.gamma_k = torch.rand(H * d, generator=g, dtype=torch.float32) + 0.5
         inp.gamma_q = torch.rand(H * d, generator=g, dtype=torch.float32) + 0.5
     return inp
+
+
+def tile_mask(w: Workload, density: float | None = None, seed: int | None = None) -> torch.Tensor:
+    """Seeded block mask, int32 [n_nodes][tiles][mask_words] (32-bit words of bits).
+
+    Bit k of row (node, query tile) is key tile k % tiles of the node's state
+    k // tiles: state 0 is the node's own chunk, state 1 + j its j-th context
+    state in selection order.  The own chunk's tiles are always kept; every
+    other bit is kept when a U(0, 1) draw (one per bit, in row-major order, on
+    a generator seeded with `seed`, default the workload's seed + 1000) is
+    below `density` (default the workload's).  Bits past a node's actual
+    context count are drawn too and ignored.
+    """
+    density = w.sparse if density is None else density
+    if density is None:
+        raise ValueError(f"workload {w.name} has no sparse density")
+    g = torch.Generator(device="cpu")
+    g.manual_seed(w.seed + 1000 if seed is None else seed)
+    nt = w.tiles
+    nbits = (1 + w.W) * nt
+    keep = torch.rand((w.n_nodes, nt, nbits), generator=g, dtype=torch.float32) < density
+    keep[:, :, :nt] = True
+    return pack_bits(keep, w.mask_words)
+
+
+def pack_bits(keep: torch.Tensor, words: int) -> torch.Tensor:
+    """bool [..., nbits] -> int32 [..., words], bit k in word k // 32 at position k % 32."""
+    nbits = keep.shape[-1]
+    pad = torch.zeros(keep.shape[:-1] + (words * 32 - nbits,), dtype=torch.bool)
+    b = torch.cat([keep, pad], dim=-1).reshape(keep.shape[:-1] + (words, 32)).to(torch.int64)
+    v = (b << torch.arange(32, dtype=torch.int64)).sum(-1)
+    return torch.where(v >= 2 ** 31, v - 2 ** 32, v).to(torch.int32)
+
+
+def unpack_bits(words: torch.Tensor, nbits: int) -> torch.Tensor:
+    """int32 [..., words] -> bool [..., nbits] (inverse of pack_bits)."""
+    v = words.to(torch.int64) & 0xFFFFFFFF
+    b = (v.unsqueeze(-1) >> torch.arange(32, dtype=torch.int64)) & 1
+    return b.reshape(words.shape[:-1] + (-1,))[..., :nbits].to(torch.bool)
 
 
 def all_states(w: Workload, inp: Inputs) -> dict:

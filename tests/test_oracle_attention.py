@@ -199,3 +199,70 @@ def test_frame_causal_single_frame_is_bidirectional(oracle_mod):
     b, lb, _ = oracle_mod.node_forward(g, 2, w.W, w.nodes[0], states, q, [0, 1], range(w.T), 0.125)
     np.testing.assert_array_equal(a, b)
     np.testing.assert_array_equal(la, lb)
+
+
+def _sparse_case(oracle_mod, within):
+    w = I.WORKLOADS["tinys"]                  # 320-token chunks: 3 tiles, the last of 64 rows
+    if within == "frame_causal":              # two latent frames of 160 tokens
+        w = I.Workload(**{**w.__dict__, "name": "tinysfc", "F": 2, "Hp": 8, "within": within})
+    inp = I.generate(w)
+    g = oracle_mod.Geometry(F=w.F, Hp=w.Hp, Wp=w.Wp, H=w.H, d=w.d, pairs=w.pairs, theta=w.theta)
+    states = {k: (_f64(a), _f64(b)) for k, (a, b) in I.all_states(w, inp).items()}
+    masks = I.unpack_bits(I.tile_mask(w), (1 + w.W) * w.tiles).numpy()
+    return w, inp, g, states, masks
+
+
+@pytest.mark.parametrize("within", ["bidirectional", "frame_causal"])
+def test_tile_mask_against_dense_brute_force(oracle_mod, within):
+    from oracle import brute
+    w, inp, g, states, masks = _sparse_case(oracle_mod, within)
+    # the brute force sees extra states the nodes must not read
+    rng = np.random.default_rng(5)
+    grid = dict(states)
+    for s in [(0, 2, 0), (0, 4, 0), (0, 1, 1)]:
+        grid[s] = (rng.standard_normal((w.T, w.H, w.d)), rng.standard_normal((w.T, w.H, w.d)))
+    scale = 1.0 / math.sqrt(w.d)
+    for i, node in enumerate(w.nodes):
+        assert not masks[i].all()             # the mask hides something for this node
+        q = _f64(inp.q[i])
+        out, lse, _ = oracle_mod.node_forward(g, oracle_mod.POLICY_IDS[w.policy], w.W, node, states,
+                                              q, range(w.H), range(w.T), scale, within=within,
+                                              tile_mask=masks[i])
+        bo, bl = brute.brute_forward(w.policy, w.W, w.F, w.Hp, w.Wp, w.pairs, w.theta, node, grid, q,
+                                     range(w.H), scale, frame_causal=within == "frame_causal",
+                                     tile_mask=masks[i])
+        np.testing.assert_allclose(out, bo, rtol=0, atol=1e-12)
+        np.testing.assert_allclose(lse, bl, rtol=0, atol=1e-12)
+        dense, _, _ = oracle_mod.node_forward(g, oracle_mod.POLICY_IDS[w.policy], w.W, node, states,
+                                              q, range(w.H), range(w.T), scale, within=within)
+        assert not np.allclose(out, dense)        # the mask changes the result
+
+
+def test_tile_mask_special_cases(oracle_mod):
+    """All bits set is the dense node; no context bit set is the node with
+    every selected state hidden; a query tile with no bit at all gets O = 0."""
+    w, inp, g, states, masks = _sparse_case(oracle_mod, "bidirectional")
+    pol = oracle_mod.POLICY_IDS[w.policy]
+    node = w.nodes[0]
+    q = _f64(inp.q[0])
+    nt = w.tiles
+    dense, dl, sel = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), range(w.T), 0.125)
+    ones = np.ones_like(masks[0])
+    a, la, _ = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), range(w.T), 0.125,
+                                       tile_mask=ones)
+    np.testing.assert_array_equal(a, dense)
+    np.testing.assert_array_equal(la, dl)
+    own_only = np.zeros_like(ones)
+    own_only[:, :nt] = True
+    b, lb, _ = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), range(w.T), 0.125,
+                                       tile_mask=own_only)
+    hid, lh, _ = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), range(w.T), 0.125,
+                                         hidden=frozenset(sel))
+    np.testing.assert_array_equal(b, hid)
+    np.testing.assert_array_equal(lb, lh)
+    none_for_tile1 = ones.copy()
+    none_for_tile1[1, :] = False
+    c, lc, _ = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), range(w.T), 0.125,
+                                       tile_mask=none_for_tile1)
+    assert np.all(c[:, 128:256] == 0.0) and np.all(lc[:, 128:256] == -np.inf)
+    np.testing.assert_array_equal(c[:, :128], dense[:, :128])
