@@ -214,6 +214,32 @@ sva_status sva_rope_kv_write_qknorm(sva_cache* c, const sva_node* nodes, int32_t
 sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* q,
                             void* out, float* lse, float scale, sva_stream s);
 
+/* sva_attend_nodes with query-dependent block-sparse access: the token-level
+ * mask M of Eq. 4 (Section 3.2), which may give every query its own subset of
+ * the causal history, taken at the granularity of 128-query x 128-key tiles.
+ *   tile_mask  device array of 32-bit words [n_nodes][nt][words_per_row],
+ *              nt = ceil(T / 128) (query tiles of a node = key tiles of a
+ *              state).  Bit k (word k / 32, bit k % 32) of row (node i, query
+ *              tile qt) set: queries [128 qt, 128 qt + 128) of node i may
+ *              attend key tile k % nt (keys [128 (k % nt), ...)) of the node's
+ *              key state k / nt, where state 0 is the own slot and state
+ *              1 + j is nodes[i].ctx_slot[j].  4-byte aligned; read by the
+ *              kernel on `s`, so it must stay valid until that completes.
+ *   words_per_row >= ceil((1 + n_ctx) * nt / 32) for every node, and
+ *              (1 + n_ctx) * nt <= 4096.
+ * The tile mask adds to every other mask: keys of hidden context slots, of
+ * later frames under SVA_WITHIN_FRAME_CAUSAL and the padding stay masked
+ * whatever the bit.  Key tiles that no query tile of a work unit (a pair of
+ * query tiles) may attend are neither loaded nor multiplied, so the cost
+ * falls with the density.  A query that sees no key gets O = 0 and LSE =
+ * -inf.  Split plans are chosen as for the dense mask.  Errors: as
+ * sva_attend_nodes, plus INVALID_ARGUMENT for a NULL or misaligned mask or a
+ * short row and CAPACITY beyond 4096 key tiles per node. */
+sva_status sva_attend_nodes_sparse(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
+                                   const void* q, void* out, float* lse, float scale,
+                                   const uint32_t* tile_mask, int32_t words_per_row,
+                                   sva_stream s);
+
 /* Bytes of the optional split workspace of a cache (0 if c is NULL).  With
  * a workspace attached, sva_attend_nodes may divide each (node, head,
  * query-tile pair) work unit into up to 4 contiguous key ranges computed by

@@ -141,12 +141,28 @@ struct Bars {
   uint64_t v_empty[4];
 };
 
+// Block-sparse launches: the first key tile at or after `from` that either
+// query tile of the unit may attend (bitmaps in the kernel's tile order), or
+// n_all if there is none.
+template <int W>
+__device__ __forceinline__ int next_tile(const uint32_t (*tm)[W], int from, int n_all) {
+  if (from >= n_all) return n_all;
+  const int words = (n_all + 31) >> 5;
+  int w = from >> 5;
+  uint32_t u = (tm[0][w] | tm[1][w]) & (~0u << (from & 31));
+  while (u == 0) {
+    if (++w >= words) return n_all;
+    u = tm[0][w] | tm[1][w];
+  }
+  return (w << 5) + __ffs(u) - 1;
+}
+
 __device__ __forceinline__ void record_timeout(const AttnParams& p, volatile int* abort_flag) {
   *abort_flag = 1;
   atomicCAS(p.status, kStatusOk, kStatusTimeout);
 }
 
-template <int D>
+template <int D, bool kSparse>
 __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_constant__ AttnParams p) {
   using C = AttnCfg<D>;
   extern __shared__ uint8_t smem_raw[];
@@ -170,10 +186,17 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
   const int h = rest / p.n_nodes;
   const AttnNode& nd = p.nodes[ni];
   const int n_all = nd.n_kv * p.nt_slot;  // key tiles of the node
-  const int t_begin = (int)((long long)split * n_all / p.n_split);
-  const int n_tiles = (int)((long long)(split + 1) * n_all / p.n_split) - t_begin;
   const int qt0 = 2 * qp;
   const bool has_q1 = qt0 + 1 < p.n_qt;
+  // Key tiles of this CTA: a contiguous range of the node's tiles, or under
+  // a block-sparse mask a contiguous range of the tiles either query tile
+  // may attend (set in the prologue below).
+  constexpr bool sparse = kSparse;  // a launch with a block-sparse tile mask
+  int t_begin = (int)((long long)split * n_all / p.n_split);
+  int n_tiles = (int)((long long)(split + 1) * n_all / p.n_split) - t_begin;
+  // per query tile, bit i = kernel key tile i (block-sparse instances only)
+  __shared__ uint32_t tmask[2][kSparse ? kMaskWords : 1];
+  __shared__ int sp_first, sp_count;
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
@@ -198,9 +221,56 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     tmem_alloc(&tmem_base_sh, C::kTmemCols);
     tmem_relinquish();
   }
+  if constexpr (sparse) if (warp == 2) {
+    // Gather the caller's mask rows of the two query tiles into the kernel's
+    // key tile order (slot list without hidden context slots), then take
+    // this split's share of the union's set bits.
+    const int words = (n_all + 31) >> 5;  // <= kMaskWords, checked on the host
+    const uint32_t* row0 = p.tile_mask + ((size_t)nd.q_index * p.n_qt + qt0) * p.mask_words;
+    const uint32_t* row1 = row0 + p.mask_words;
+    int total = 0;
+    for (int w = 0; w < words; ++w) {
+      const int i = (w << 5) + lane;
+      bool b0 = false, b1 = false;
+      if (i < n_all) {
+        const int s = i / p.nt_slot;
+        const int k = nd.src[s] * p.nt_slot + (i - s * p.nt_slot);
+        b0 = (row0[k >> 5] >> (k & 31)) & 1u;
+        if (has_q1) b1 = (row1[k >> 5] >> (k & 31)) & 1u;
+      }
+      const uint32_t m0 = __ballot_sync(0xffffffffu, b0);
+      const uint32_t m1 = __ballot_sync(0xffffffffu, b1);
+      if (lane == 0) {
+        tmask[0][w] = m0;
+        tmask[1][w] = m1;
+      }
+      total += __popc(m0 | m1);
+    }
+    if (lane == 0) {
+      const int lo = (int)((long long)split * total / p.n_split);
+      const int hi = (int)((long long)(split + 1) * total / p.n_split);
+      int first = n_all, seen = 0;
+      for (int w = 0; hi > lo && w < words; ++w) {
+        uint32_t u = tmask[0][w] | tmask[1][w];
+        const int cnt = __popc(u);
+        if (seen + cnt > lo) {
+          for (int r = lo - seen; r > 0; --r) u &= u - 1;  // drop the bits before the lo-th
+          first = (w << 5) + __ffs(u) - 1;
+          break;
+        }
+        seen += cnt;
+      }
+      sp_first = first;
+      sp_count = hi - lo;
+    }
+  }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if constexpr (sparse) {
+    t_begin = sp_first;
+    n_tiles = sp_count;
+  }
   const uint32_t tbase = tmem_base_sh;
   const uint64_t tmo = p.timeout_ns;
 
@@ -227,8 +297,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
                       (qt0 + 1) * kTile, nd.q_index);
       }
       const uint64_t keep = l2_policy_evict_last();
-      for (int j = 0; j < n_tiles; ++j) {
-        const int i = t_begin + j;  // key tile of the node
+      int i = t_begin;  // key tile of the node
+      for (int j = 0; j < n_tiles; ++j, i = sparse ? next_tile(tmask, i + 1, n_all) : i + 1) {
         const int ks = j % C::kKStages;
         const int vs = j % C::kVStages;
         const int slot = nd.slot[i / p.nt_slot];
@@ -280,15 +350,25 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       const uint64_t dK = sdesc_sw128(smem_u32(sK), 16, 1024);
       const uint64_t dV = sdesc_sw128(smem_u32(sV), C::kBoxBytes, 1024);
       constexpr uint64_t kTileStep = (uint64_t)(C::kTileBytes >> 4);
+      // Under a block-sparse mask a query tile may skip a key tile the other
+      // query tile attends: its S and PV MMAs are then not issued (the S
+      // barrier is still committed, so every barrier completes once per
+      // tile), and its first issued PV starts the accumulator.
+      auto vis = [&](int b, int kt) {
+        return !sparse || ((tmask[b][kt >> 5] >> (kt & 31)) & 1u) != 0u;
+      };
+      bool pv_started[2] = {false, false};
       // S_b = Q_b K_i^T into TMEM buffer b
-      auto issue_s = [&](int b, int i) {
-        const uint64_t kb = dK + (uint64_t)(i % C::kKStages) * kTileStep;
-        const uint64_t qb = dQ[b];
-        const uint32_t dcol = tbase + col_s(b);
+      auto issue_s = [&](int b, int i, bool v) {
+        if (v) {
+          const uint64_t kb = dK + (uint64_t)(i % C::kKStages) * kTileStep;
+          const uint64_t qb = dQ[b];
+          const uint32_t dcol = tbase + col_s(b);
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint64_t off = (uint64_t)(((kk >> 2) * C::kBoxBytes + (kk & 3) * 32) >> 4);
-          mma_ss_warp(dcol, qb + off, kb + off, idesc_qk, kk > 0 ? 1u : 0u);
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint64_t off = (uint64_t)(((kk >> 2) * C::kBoxBytes + (kk & 3) * 32) >> 4);
+            mma_ss_warp(dcol, qb + off, kb + off, idesc_qk, kk > 0 ? 1u : 0u);
+          }
         }
         mma_commit_warp(&bars.s_full[b]);
       };
@@ -297,11 +377,12 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         const uint64_t vb = dV + (uint64_t)(i % C::kVStages) * kTileStep;
         const uint32_t ocol = tbase + col_o(b);
         const uint32_t pcol = tbase + col_s(b);
-        const uint32_t acc0 = i > 0 ? 1u : 0u;
+        const uint32_t acc0 = (sparse ? pv_started[b] : i > 0) ? 1u : 0u;
 #pragma unroll
         for (int kk = 0; kk < kTile / 16; ++kk)
           mma_ts_warp(ocol, pcol + kk * 8, vb + (uint64_t)((kk * 2048) >> 4), idesc_pv,
                  kk > 0 ? 1u : acc0);
+        if (sparse) pv_started[b] = true;
       };
       auto wait = [&](uint64_t* bar, uint32_t parity) {
         return __all_sync(0xffffffffu, mbar_wait(bar, parity, &abort_flag, tmo));
@@ -310,15 +391,19 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         return wait(&bars.k_full[i % C::kKStages], (uint32_t)(i / C::kKStages) & 1u);
       };
       bool ok = wait(&bars.q_full, 0);
-      ok = ok && wait_k(0);
-      if (ok) {
-        tc_fence_after();
-        issue_s(0, 0);
-        if (has_q1) issue_s(1, 0);
+      int kt = t_begin;  // key tile of the node at iteration i
+      if (n_tiles > 0) {  // a block-sparse range may be empty: then only o_final is committed
+        ok = ok && wait_k(0);
+        if (ok) {
+          tc_fence_after();
+          issue_s(0, 0, vis(0, kt));
+          if (has_q1) issue_s(1, 0, vis(1, kt));
+        }
       }
       for (int i = 0; ok && i < n_tiles; ++i) {
         const uint32_t par = (uint32_t)i & 1u;
         const bool more = i + 1 < n_tiles;
+        const int kt_next = !more ? kt : (sparse ? next_tile(tmask, kt + 1, n_all) : kt + 1);
         // V_i and K_{i+1} land long before the softmax hands over P_0, so
         // their waits go first, off the path from P_0 to the next MMA.
         if (!wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u) ||
@@ -327,17 +412,18 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
           break;
         }
         tc_fence_after();
-        issue_pv(0, i);
-        if (more) issue_s(0, i + 1);
+        if (vis(0, kt)) issue_pv(0, i);
+        if (more) issue_s(0, i + 1, vis(0, kt_next));
         if (has_q1) {
           if (!wait(&bars.p_full[1], par)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          issue_pv(1, i);
+          if (vis(1, kt)) issue_pv(1, i);
         }
-        if (more && has_q1) issue_s(1, i + 1);
+        if (more && has_q1) issue_s(1, i + 1, vis(1, kt_next));
+        kt = kt_next;
       }
       if (ok) {
         mma_commit_warp(&bars.o_final);
@@ -395,6 +481,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     const float sl2 = p.scale_log2;
     const uint64_t sl2x2 = f2u(sl2, sl2);
     const int frame_causal = nd.frame_causal;
+    bool o_has[2] = {false, false};       // O_b holds a PV (some key tile was attended)
     float m[2] = {-INFINITY, -INFINITY};  // running max of scale*log2(e)*logit per query tile
     float l[2] = {0.0f, 0.0f};            // this thread's part of the running sum of 2^(x - m)
     // first token of the latent frame after this row's (frame-causal mask)
@@ -410,10 +497,11 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     // it about as long as an MMA issue).
     const bool releaser = warp == 4 && lane == 0;
     bool ok = true;
-    for (int i = 0; ok && i < n_tiles; ++i) {
-      const int t = (t_begin + i) % p.nt_slot;  // key tile inside its slot
+    int kt = t_begin;  // key tile of the node
+    for (int i = 0; ok && i < n_tiles; ++i, kt = sparse ? next_tile(tmask, kt + 1, n_all) : kt + 1) {
+      const int t = kt % p.nt_slot;  // key tile inside its slot
       const int valid_tile = (t == p.nt_slot - 1) ? p.valid_last : kTile;
-      const bool own_fc = frame_causal && t_begin + i < p.nt_slot;
+      const bool own_fc = frame_causal && kt < p.nt_slot;
 #pragma unroll
       for (int b = 0; b < 2; ++b) {
         if (b == 1 && !has_q1) break;
@@ -423,6 +511,11 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         if (releaser && b == nb - 1) {
           mbar_arrive(&bars.k_empty[i % C::kKStages]);
           if (i > 0) mbar_arrive(&bars.v_empty[(i - 1) % C::kVStages]);
+        }
+        if (sparse && !((tmask[b][kt >> 5] >> (kt & 31)) & 1u)) {
+          // query tile b skips this key tile: no S was computed, no P is due
+          mbar_arrive(&bars.p_full[b]);
+          continue;
         }
         tc_fence_after();
         const uint32_t scol = tbase + lane_off + col_s(b);
@@ -467,9 +560,9 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         const bool need = m_new > m[b] + kRescaleThreshold;
         if (__any_sync(0xffffffffu, need)) {
           const float alpha = ex2(m[b] - m_new);  // 0 on the first tile (m = -inf)
-          if (i > 0) {
-            // O_b holds the sum over tiles < i: the commit that completed S_b
-            // of tile i came after PV_b of tile i-1.
+          if (sparse ? o_has[b] : i > 0) {
+            // O_b holds the sum over earlier tiles: the commit that completed
+            // S_b of this tile came after PV_b of the previous one.
 #pragma unroll
             for (int c = 0; c < DH / 32; ++c) {
               uint32_t o[32];
@@ -516,6 +609,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         tmem_wait_st();
         tc_fence_before();
         mbar_arrive(&bars.p_full[b]);
+        if (sparse) o_has[b] = true;
       }
     }
     if (ok) {
@@ -540,8 +634,13 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
 #pragma unroll
           for (int c = 0; c < DH / 32; ++c) {
             uint32_t o[32];
-            tmem_ld16x2_32<DH>(tbase + lane_off + col_o(b) + c * 32, o);
-            tmem_wait_ld(o);
+            if (!sparse || o_has[b]) {  // dense ranges are never empty
+              tmem_ld16x2_32<DH>(tbase + lane_off + col_o(b) + c * 32, o);
+              tmem_wait_ld(o);
+            } else {  // no key tile attended in this range (block-sparse): no MMA wrote O
+#pragma unroll
+              for (int e = 0; e < 32; ++e) o[e] = 0u;
+            }
             if (in_range) {
               uint4* dst = reinterpret_cast<uint4*>(orow + c * 32);
 #pragma unroll
@@ -576,8 +675,13 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
 #pragma unroll
           for (int c = 0; c < DH / 32; ++c) {
             uint32_t o[32];
-            tmem_ld16x2_32<DH>(tbase + lane_off + col_o(b) + c * 32, o);
-            tmem_wait_ld(o);
+            if (!sparse || o_has[b]) {  // dense ranges are never empty
+              tmem_ld16x2_32<DH>(tbase + lane_off + col_o(b) + c * 32, o);
+              tmem_wait_ld(o);
+            } else {  // no key tile attended in this range (block-sparse): no MMA wrote O
+#pragma unroll
+              for (int e = 0; e < 32; ++e) o[e] = 0u;
+            }
 #pragma unroll
             for (int v = 0; v < 8; ++v)
               part4[(DH * half / 4 + c * 8 + v) * 256 + r] =
@@ -677,20 +781,26 @@ cudaError_t launch_d(const AttnParams& p, int grid, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (!configured[dev]) {
-    e = cudaFuncSetAttribute(attend_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             C::kSmemBytes);
-    if (e != cudaSuccess) return e;
+    for (auto k : {attend_kernel<D, false>, attend_kernel<D, true>}) {
+      e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+      if (e != cudaSuccess) return e;
+    }
     // setmaxnreg.inc waits until the block's register pool can serve it: a
     // build whose launch register count leaves the split short would never
     // proceed, so such a build is refused here.
-    cudaFuncAttributes fa;
-    e = cudaFuncGetAttributes(&fa, attend_kernel<D>);
-    if (e != cudaSuccess) return e;
-    if (fa.numRegs * kThreads < 4 * 32 * kRegsLow + 8 * 32 * kRegsHigh)
-      return cudaErrorInvalidConfiguration;
+    for (auto k : {attend_kernel<D, false>, attend_kernel<D, true>}) {
+      cudaFuncAttributes fa;
+      e = cudaFuncGetAttributes(&fa, k);
+      if (e != cudaSuccess) return e;
+      if (fa.numRegs * kThreads < 4 * 32 * kRegsLow + 8 * 32 * kRegsHigh)
+        return cudaErrorInvalidConfiguration;
+    }
     configured[dev] = true;
   }
-  attend_kernel<D><<<grid, kThreads, C::kSmemBytes, s>>>(p);
+  if (p.tile_mask != nullptr)
+    attend_kernel<D, true><<<grid, kThreads, C::kSmemBytes, s>>>(p);
+  else
+    attend_kernel<D, false><<<grid, kThreads, C::kSmemBytes, s>>>(p);
   return cudaGetLastError();
 }
 

@@ -14,6 +14,7 @@ namespace sva {
 constexpr int kTile = 128;  // query rows per Q tile and key rows per K/V tile
 constexpr int kMaxSplit = 4;  // key-range splits of one work unit
 constexpr uint64_t kDefaultWaitTimeoutNs = 1000000000ull;  // bounded device waits: 1 s
+constexpr int kMaskWords = 128;  // block-sparse launches: at most 32 * 128 key tiles per node
 
 // Device status word values (a subset of sva_status).
 constexpr int kStatusOk = 0;
@@ -26,6 +27,9 @@ struct AttnNode {
   int32_t n_kv;
   int32_t frame_causal;  // own-chunk keys of later latent frames masked
   int32_t slot[1 + SVA_MAX_CTX];
+  // key state (0 = own, 1 + j = the caller's ctx_slot[j]) of each entry of
+  // `slot`: the row index of its tiles in a block-sparse tile mask
+  uint8_t src[1 + SVA_MAX_CTX];
 };
 
 struct alignas(128) AttnParams {
@@ -49,6 +53,8 @@ struct alignas(128) AttnParams {
   float* ws;            // split partials [unit][split][(d + 2) * 256] fp32, or null
   int* ws_count;        // per-unit arrival counters, zero between launches, or null
   uint64_t timeout_ns;
+  const uint32_t* tile_mask;  // block-sparse visibility [n_nodes][n_qt][mask_words], or null
+  int32_t mask_words;
   AttnNode nodes[SVA_MAX_NODES];
 };
 

@@ -554,8 +554,15 @@ sva_status sva_rope_kv_write_qknorm(sva_cache* c, const sva_node* nodes, int32_t
   return rope_write(c, nodes, n_nodes, k_new, v_new, q_inout, gamma_k, gamma_q, eps, s);
 }
 
-sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* q,
-                            void* out, float* lse, float scale, sva_stream s) {
+}  // extern "C"
+
+namespace {
+
+// sva_attend_nodes and sva_attend_nodes_sparse: the checks and the launch;
+// tile_mask NULL is the dense mask.
+sva_status attend(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* q, void* out,
+                  float* lse, float scale, const uint32_t* tile_mask, int32_t mask_words,
+                  sva_stream s) {
   if (c == nullptr || nodes == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "NULL argument");
   if (n_nodes < 1) return fail(SVA_ERR_INVALID_ARGUMENT, "n_nodes %d < 1", n_nodes);
   if (n_nodes > SVA_MAX_NODES)
@@ -583,6 +590,7 @@ sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes
     a.q_index = i;
     a.frame_causal = n.within == SVA_WITHIN_FRAME_CAUSAL ? 1 : 0;
     a.slot[0] = n.own_slot;
+    a.src[0] = 0;
     int nkv = 1;
     for (int k = 0; k < n.n_ctx; ++k) {
       const int32_t cs = n.ctx_slot[k];
@@ -602,9 +610,30 @@ sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes
       for (int k2 = 0; k2 < k; ++k2)
         if (n.ctx_slot[k2] == cs)
           return fail(SVA_ERR_INVALID_ARGUMENT, "node %d: slot %d listed twice", i, cs);
-      if (n.ctx_visible[k]) a.slot[nkv++] = cs;
+      if (n.ctx_visible[k]) {
+        a.src[nkv] = (uint8_t)(1 + k);
+        a.slot[nkv++] = cs;
+      }
     }
     a.n_kv = nkv;
+  }
+  p.n_qt = (c->L.T + sva::kTile - 1) / sva::kTile;
+  p.nt_slot = c->L.Tpad / sva::kTile;
+  if (tile_mask != nullptr) {
+    if ((reinterpret_cast<uintptr_t>(tile_mask) & 3u) != 0)
+      return fail(SVA_ERR_INVALID_ARGUMENT, "tile_mask must be 4-byte aligned");
+    for (int i = 0; i < n_nodes; ++i) {
+      const long long bits = (long long)(1 + nodes[i].n_ctx) * p.nt_slot;
+      if (bits > 32LL * sva::kMaskWords)
+        return fail(SVA_ERR_CAPACITY, "node %d: %lld key tiles exceed the %d a tile mask covers",
+                    i, bits, 32 * sva::kMaskWords);
+      if (mask_words < (bits + 31) / 32)
+        return fail(SVA_ERR_INVALID_ARGUMENT,
+                    "node %d: words_per_row %d < %lld needed for %lld key tiles", i, mask_words,
+                    (bits + 31) / 32, bits);
+    }
+    p.tile_mask = tile_mask;
+    p.mask_words = mask_words;
   }
   if (c->q_cached != q || c->q_cached_n != n_nodes) {
     st = encode_4d_q(&c->tmap_q, q, g, c->L.T, n_nodes);
@@ -624,10 +653,8 @@ sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes
   p.T = c->L.T;
   p.Tpad = c->L.Tpad;
   p.H = g.num_heads;
-  p.n_qt = (c->L.T + sva::kTile - 1) / sva::kTile;
   p.n_qp = (p.n_qt + 1) / 2;
   p.n_nodes = n_nodes;
-  p.nt_slot = c->L.Tpad / sva::kTile;
   p.valid_last = c->L.T - (p.nt_slot - 1) * sva::kTile;
   p.frame_tokens = g.grid_h * g.grid_w;
   p.fault_mode = c->fault_mode;
@@ -645,6 +672,23 @@ sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes
   cudaError_t e = sva::launch_attend(p, g.head_dim, (int)grid, reinterpret_cast<cudaStream_t>(s));
   if (e != cudaSuccess) return cuda_fail(e, "attend launch");
   return ok();
+}
+
+}  // namespace
+
+extern "C" {
+
+sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* q,
+                            void* out, float* lse, float scale, sva_stream s) {
+  return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, s);
+}
+
+sva_status sva_attend_nodes_sparse(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
+                                   const void* q, void* out, float* lse, float scale,
+                                   const uint32_t* tile_mask, int32_t words_per_row,
+                                   sva_stream s) {
+  if (tile_mask == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "tile_mask is NULL");
+  return attend(c, nodes, n_nodes, q, out, lse, scale, tile_mask, words_per_row, s);
 }
 
 // Attention with the split scratch taken from the library's own device

@@ -52,6 +52,7 @@ class Workload:
     within: str = "bidirectional"  # visibility inside the own chunk (or "frame_causal")
     qknorm: bool = False  # RMS-normalise K and Q per token before RoPE (seeded gammas)
     sparse: float | None = None  # density of kept context key tiles (block-sparse mask), or None
+    sparse_rows: int = 1  # consecutive query tiles sharing one mask row (draws per group)
     description: str = ""
     theta: float = 10000.0
     pairs: tuple = field(default=None)
@@ -151,8 +152,9 @@ WORKLOADS = {
     "prog4s": Workload(
         name="prog4s", seed=9, F=3, Hp=30, Wp=52, H=12, d=128, K=4, W=6, policy="prog",
         nodes=_round_nodes(0, 4, 20), prefilled=_PROG_PREFILL_20, round=20, sparse=0.5,
-        description="prog4 with query-dependent block-sparse access: every query tile keeps its "
-                    "own chunk and a seeded half of the 128-token key tiles of its history"),
+        sparse_rows=2,
+        description="prog4 with query-dependent block-sparse access: every 256-query block keeps "
+                    "its own chunk and a seeded half of the 128-token key tiles of its history"),
     "prog4fc": Workload(
         name="prog4fc", seed=8, F=3, Hp=30, Wp=52, H=12, d=128, K=4, W=6, policy="prog",
         nodes=_round_nodes(0, 4, 20), prefilled=_PROG_PREFILL_20, round=20,
@@ -220,8 +222,9 @@ def tile_mask(w: Workload, density: float | None = None, seed: int | None = None
     state in selection order.  The own chunk's tiles are always kept; every
     other bit is kept when a U(0, 1) draw (one per bit, in row-major order, on
     a generator seeded with `seed`, default the workload's seed + 1000) is
-    below `density` (default the workload's).  Bits past a node's actual
-    context count are drawn too and ignored.
+    below `density` (default the workload's).  With `sparse_rows` = r > 1 the
+    draws are made for groups of r consecutive query tiles, which share one
+    row.  Bits past a node's actual context count are drawn too and ignored.
     """
     density = w.sparse if density is None else density
     if density is None:
@@ -230,7 +233,10 @@ def tile_mask(w: Workload, density: float | None = None, seed: int | None = None
     g.manual_seed(w.seed + 1000 if seed is None else seed)
     nt = w.tiles
     nbits = (1 + w.W) * nt
-    keep = torch.rand((w.n_nodes, nt, nbits), generator=g, dtype=torch.float32) < density
+    r = w.sparse_rows
+    groups = -(-nt // r)
+    keep = torch.rand((w.n_nodes, groups, nbits), generator=g, dtype=torch.float32) < density
+    keep = keep.repeat_interleave(r, dim=1)[:, :nt]
     keep[:, :, :nt] = True
     return pack_bits(keep, w.mask_words)
 

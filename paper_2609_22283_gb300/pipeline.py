@@ -9,7 +9,9 @@ serial node, Eq. 5):
   3. the fused 3D-RoPE + cache scatter of the nodes' new K/V and in-place Q
      rotation (sva_rope_kv_write), which also makes this round's states
      readable by the progressive nodes of the same round (Section 3.3);
-  4. the batched policy-indexed attention (sva_attend_nodes, Eq. 4).
+  4. the batched policy-indexed attention (sva_attend_nodes, Eq. 4; with a
+     block-sparse workload sva_attend_nodes_sparse and the workload's seeded
+     key-tile mask).
 Steps 3 and 4 are stream-ordered kernels; 1 and 2 are host integer work.
 """
 from __future__ import annotations
@@ -19,7 +21,7 @@ import math
 import torch
 
 from . import sva
-from .inputs import Inputs, Workload
+from .inputs import Inputs, Workload, tile_mask
 
 
 def geometry_for(w: Workload, spare_slots: int = 2) -> sva.sva_geometry:
@@ -39,6 +41,7 @@ class Step:
             self.cache.set_workspace(ws)
         self.own = {}
         self.scale = 1.0 / math.sqrt(w.d)
+        self.mask = tile_mask(w).to(self.device) if w.sparse is not None else None
 
     def prefill(self, inp: Inputs, stream=None):
         """Binds and writes the workload's history states (untimed set-up)."""
@@ -88,8 +91,16 @@ class Step:
         else:
             self.cache.rope_kv_write(nodes, k_new, v_new, q if rotate_q else None, stream=stream,
                                      check=False)
-        self.cache.attend_nodes(nodes, q, out, lse, self.scale, stream=stream, check=False)
+        self.attend(nodes, q, out, lse, stream=stream)
         return n
+
+    def attend(self, nodes, q, out, lse=None, stream=None):
+        """Step 4 alone (dense or block-sparse, as the workload says)."""
+        if self.mask is not None:
+            self.cache.attend_nodes_sparse(nodes, q, out, self.mask, lse, self.scale, stream=stream,
+                                           check=False)
+        else:
+            self.cache.attend_nodes(nodes, q, out, lse, self.scale, stream=stream, check=False)
 
     def device_inputs(self, inp: Inputs):
         d = self.device

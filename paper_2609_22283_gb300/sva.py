@@ -38,7 +38,7 @@ MAX_NODES = 64
 EXPORTED = ("sva_cache_bytes", "sva_cache_create", "sva_cache_bind", "sva_cache_lookup",
             "sva_cache_release", "sva_select_context", "sva_pipeline_round", "sva_check_pipeline",
             "sva_rope_kv_write", "sva_rope_kv_write_qknorm", "sva_attend_nodes",
-            "sva_attend_workspace_bytes",
+            "sva_attend_nodes_sparse", "sva_attend_workspace_bytes",
             "sva_cache_set_workspace", "sva_attend_nodes_noalloc", "sva_poll_device_status",
             "sva_debug_inject", "sva_destroy", "sva_last_error")
 
@@ -90,6 +90,7 @@ def load(path: str = LIB_PATH):
         "sva_rope_kv_write": ([p, pn, i32, p, p, p, p], i32),
         "sva_rope_kv_write_qknorm": ([p, pn, i32, p, p, p, p, p, ctypes.c_float, p], i32),
         "sva_attend_nodes": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
+        "sva_attend_nodes_sparse": ([p, pn, i32, p, p, p, ctypes.c_float, p, i32, p], i32),
         "sva_attend_workspace_bytes": ([p], ctypes.c_size_t),
         "sva_attend_nodes_noalloc": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
         "sva_cache_set_workspace": ([p, p, ctypes.c_size_t], i32),
@@ -281,6 +282,34 @@ class Cache:
                                    ctypes.c_void_p(out.data_ptr()),
                                    ctypes.c_void_p(lse.data_ptr() if lse is not None else 0),
                                    float(scale), ctypes.c_void_p(_stream_handle(stream)))
+        _check(st)
+
+    def attend_nodes_sparse(self, nodes, q, out, tile_mask, lse=None, scale=None, stream=None,
+                            check=True):
+        """sva_attend_nodes_sparse: tile_mask is a contiguous int32 CUDA tensor
+        [n_nodes][ceil(T/128)][words] of key-tile bits (see include/sva.h)."""
+        n = len(nodes) if not isinstance(nodes, ctypes.Array) else None
+        arr = nodes if isinstance(nodes, ctypes.Array) else make_nodes(nodes)
+        count = n if n is not None else len(arr)
+        g = self.g
+        nt = -(-self.T // 128)
+        if check:
+            _tok_major(q, "q", count, self.T, g.num_heads, g.head_dim)
+            _tok_major(out, "out", count, self.T, g.num_heads, g.head_dim)
+            if lse is not None and (lse.dtype != torch.float32 or not lse.is_contiguous()
+                                    or tuple(lse.shape) != (count, g.num_heads, self.T)):
+                raise ValueError("lse must be a contiguous fp32 tensor [n][H][T]")
+        if (tile_mask.dtype != torch.int32 or not tile_mask.is_cuda or not tile_mask.is_contiguous()
+                or tile_mask.dim() != 3 or tuple(tile_mask.shape[:2]) != (count, nt)):
+            raise ValueError(f"tile_mask must be a contiguous int32 CUDA tensor [{count}][{nt}][words]")
+        if scale is None:
+            scale = 1.0 / math.sqrt(g.head_dim)
+        st = _lib.sva_attend_nodes_sparse(self.handle, arr, count, ctypes.c_void_p(q.data_ptr()),
+                                          ctypes.c_void_p(out.data_ptr()),
+                                          ctypes.c_void_p(lse.data_ptr() if lse is not None else 0),
+                                          float(scale), ctypes.c_void_p(tile_mask.data_ptr()),
+                                          int(tile_mask.shape[2]),
+                                          ctypes.c_void_p(_stream_handle(stream)))
         _check(st)
 
     def workspace_bytes(self) -> int:
