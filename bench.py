@@ -41,8 +41,23 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 
 
 def attn_flops(w) -> float:
-    """Algorithmic FLOPs of one step's attention: 4*T*Lkv*d*H per node (QK^T + PV)."""
+    """Algorithmic FLOPs of one step's attention: 4*T*Lkv*d*H per node (QK^T + PV).
+    With a block-sparse mask only the (query tile, key tile) pairs the mask
+    keeps count, each as 4 * rows * keys * d * H (ragged last tiles included
+    at their true size)."""
     total = 0.0
+    if w.sparse is not None:
+        from paper_2609_22283_gb300 import inputs as I
+        nt = w.tiles
+        keep = I.unpack_bits(I.tile_mask(w), (1 + w.W) * nt).numpy()
+        size = [min(128, w.T - 128 * t) for t in range(nt)]
+        for i, (_, b, _) in enumerate(w.nodes):
+            n_ctx = max(0, min(w.W, b - 1))
+            for qt in range(nt):
+                for k in range((1 + n_ctx) * nt):
+                    if keep[i, qt, k]:
+                        total += 4.0 * size[qt] * size[k % nt] * w.d * w.H
+        return total
     for (_, b, _) in w.nodes:
         n_ctx = max(0, min(w.W, b - 1))
         total += 4.0 * w.T * (1 + n_ctx) * w.T * w.d * w.H
@@ -250,6 +265,10 @@ def config_of(w, world):
     return {"workload": w.name, "description": w.description, "nodes": [list(n) for n in w.nodes],
             "policy": w.policy, "heads": w.H, "head_dim": w.d, "tokens_per_chunk": w.T,
             "kv_tokens_per_node": lkv, "window_chunks": w.W, "levels": w.K,
+            "within_chunk": w.within,
+            "block_sparse": (None if w.sparse is None else
+                             {"density": w.sparse, "query_tiles_per_row": w.sparse_rows,
+                              "flops": "kept (query tile, key tile) pairs only"}),
             "l2": "flushed between timed steps (256 MiB write, outside the timed intervals)",
             "parallelism": "single GPU" if world == 1 else f"{world} independent replicas"}
 
@@ -282,7 +301,7 @@ def run_ours(args, world, rank, local):
     def one_step():
         nodes_, _ = step.node_table()            # steps 1-2: selection + Eq. 7 check
         step.cache.rope_kv_write(nodes_, k, v, q, check=False)
-        step.cache.attend_nodes(nodes_, q, out, lse, step.scale, check=False)
+        step.attend(nodes_, q, out, lse)             # dense or block-sparse, per workload
 
     for _ in range(args.warmup):
         one_step()
@@ -301,7 +320,7 @@ def run_ours(args, world, rank, local):
             ev[i][0].record(stream)
             step.cache.rope_kv_write(nodes_, k, v, q, check=False)
             ev[i][1].record(stream)
-            step.cache.attend_nodes(nodes_, q, out, lse, step.scale, check=False)
+            step.attend(nodes_, q, out, lse)
             ev[i][2].record(stream)
         torch.cuda.synchronize()
         barrier(world)
