@@ -375,9 +375,66 @@ def run_ours(args, world, rank, local):
         torch.cuda.synchronize()
         if it >= args.warmup:
             e2e_ms.append(e0.elapsed_time(e1))
-    e2e_step = reduce_max(sum(e2e_ms) / len(e2e_ms), world)
+    e2e_serial = reduce_max(sum(e2e_ms) / len(e2e_ms), world)
     h2d = (hq.numel() + hk.numel() + hv.numel()) * 2
     d2h = hout.numel() * 2
+
+    # End to end as a caller streams steps: step i's inputs go up on one
+    # stream while step i-1 computes on another and step i-2's output comes
+    # back on a third (two device buffer sets, ordered by events).  Every step
+    # still copies its inputs from pinned host memory and its output back;
+    # the timed region runs from the first copy up to the last copy down.
+    # No L2 flush here: a step's working set (the cache it reads plus its
+    # inputs and output) exceeds the 129 MB L2.
+    s_up, s_cmp, s_down = (torch.cuda.Stream(dev) for _ in range(3))
+    bufs = [(q, k, v, out, lse)] + [tuple(torch.empty_like(t) for t in (q, k, v, out, lse))]
+    houts = [hout, torch.empty_like(hout, pin_memory=True)]
+    up_done = [torch.cuda.Event() for _ in range(2)]
+    cmp_done = [torch.cuda.Event() for _ in range(2)]
+    down_done = [torch.cuda.Event() for _ in range(2)]
+
+    def streamed(K):
+        for i in range(K):
+            bi = i % 2
+            qb, kb, vb, ob, lb = bufs[bi]
+            with torch.cuda.stream(s_up):
+                if i >= 2:
+                    s_up.wait_event(cmp_done[bi])        # step i-2 has read this buffer set
+                qb.copy_(hq, non_blocking=True)
+                kb.copy_(hk, non_blocking=True)
+                vb.copy_(hv, non_blocking=True)
+                up_done[bi].record(s_up)
+            with torch.cuda.stream(s_cmp):
+                s_cmp.wait_event(up_done[bi])
+                if i >= 2:
+                    s_cmp.wait_event(down_done[bi])      # step i-2's output has left
+                nodes_, _ = step.node_table()
+                step.cache.rope_kv_write(nodes_, kb, vb, qb, stream=s_cmp, check=False)
+                step.attend(nodes_, qb, ob, lb, stream=s_cmp)
+                cmp_done[bi].record(s_cmp)
+            with torch.cuda.stream(s_down):
+                s_down.wait_event(cmp_done[bi])
+                houts[bi].copy_(ob, non_blocking=True)
+                down_done[bi].record(s_down)
+
+    streamed(args.warmup + 2)
+    torch.cuda.synchronize()
+    k_e2e = max(4, min(args.steps, 200))
+    e_start = torch.cuda.Event(enable_timing=True)
+    e_end = torch.cuda.Event(enable_timing=True)
+    barrier(world)
+    e_start.record(s_up)
+    s_cmp.wait_event(e_start)
+    s_down.wait_event(e_start)
+    streamed(k_e2e)
+    s_down.wait_stream(s_cmp)
+    e_end.record(s_down)
+    torch.cuda.synchronize()
+    barrier(world)
+    e2e_step = reduce_max(e_start.elapsed_time(e_end) / k_e2e, world)
+    status = step.cache.poll()
+    if status != 0:
+        raise RuntimeError(f"device status {status} in the end-to-end region")
 
     peaks, peak_src = load_peaks()
     peak = peaks.get("bf16_tflops", FALLBACK_PEAKS["bf16_tflops"])
@@ -397,7 +454,12 @@ def run_ours(args, world, rank, local):
                      if peak_src == "measured" else "fallback 1.9 PFLOP/s",
                      "traffic": traffic},
         "e2e": {"value": flops * world / (e2e_step * 1e-3) / 1e12, "unit": "TFLOP/s",
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": e2e_step, "steps": k_e2e,
+                "mode": "streamed: copy-up, compute and copy-down of consecutive steps on three "
+                        "streams, two device buffer sets",
+                "serial_value": flops * world / (e2e_serial * 1e-3) / 1e12,
+                "serial_note": "each step alone: copy up, compute, copy down, synchronise"},
         "gpu_launches": 2 * args.steps,
         "clocks": clocks,
     }
