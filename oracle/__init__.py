@@ -12,6 +12,7 @@ rows) and is driven from here:
 * ``select`` / ``pipeline_round`` / ``available`` -- Eq. 2-3, Eq. 6, Eq. 7.
 * ``rope_head`` / ``bf16`` -- the 3D RoPE reading and the bf16 cache store.
 * ``attend_rows`` -- Eq. 4 masked softmax attention.
+* ``qkv_project`` -- the input projection producing q, k, v token-major.
 * ``node_forward`` -- one denoising node end to end: its context selection,
   the rotation of every key state it reads and of its queries, the bf16
   rounding of what the cache would hold, and the attention of the requested
@@ -169,6 +170,29 @@ def rms_norm(x: np.ndarray, gamma: np.ndarray, eps: float) -> np.ndarray:
     y = np.empty_like(x2)
     _load().oracle_rms_norm(_pd(x2), _pd(g), _pd(y), x2.shape[0], x2.shape[1], float(eps))
     return y.reshape(shape)
+
+
+# ---------------------------------------------------------------- QKV projection
+
+def qkv_project(x: np.ndarray, weight: np.ndarray, bias=None, heads: int = 1):
+    """The linear projection in front of the attention layer, fp64:
+    y = x W^T + b over the last axis, then split into q, k, v.
+
+    x: [rows][C]; weight: [3 * N][C] (out_features x in_features, the rows of
+    q's outputs first, then k's, then v's); bias: [3 * N] or None.
+    Returns (q, k, v), each [rows][heads][N / heads], unrounded.  A library
+    matrix product is the one step (no blocking or reordering of its own).
+    """
+    x = np.asarray(x, dtype=np.float64)
+    w = np.asarray(weight, dtype=np.float64)
+    rows, C = x.shape
+    assert w.shape[1] == C and w.shape[0] % 3 == 0
+    n = w.shape[0] // 3
+    assert n % heads == 0
+    y = x @ w.T
+    if bias is not None:
+        y = y + np.asarray(bias, dtype=np.float64)[None, :]
+    return tuple(y[:, t * n:(t + 1) * n].reshape(rows, heads, n // heads) for t in range(3))
 
 
 # ---------------------------------------------------------------- attention

@@ -257,6 +257,22 @@ def unpack_bits(words: torch.Tensor, nbits: int) -> torch.Tensor:
     return b.reshape(words.shape[:-1] + (-1,))[..., :nbits].to(torch.bool)
 
 
+def projection_inputs(w: Workload, in_features: int, seed: int | None = None):
+    """Seeded inputs of the QKV projection of a workload's nodes:
+    x [n_nodes][T][in_features] bf16 ~ N(0, 1); weight [3*H*d][in_features]
+    bf16 ~ N(0, 1/in_features) (rows: q's outputs, then k's, then v's); bias
+    [3*H*d] fp32 ~ N(0, 0.1^2); drawn in that order on a generator seeded with
+    `seed` (default the workload's seed + 2000).  Random weights stand in for
+    trained ones: the projection's cost and numerics do not depend on them."""
+    g = torch.Generator(device="cpu")
+    g.manual_seed(w.seed + 2000 if seed is None else seed)
+    n_out = 3 * w.H * w.d
+    x = torch.randn((w.n_nodes, w.T, in_features), generator=g, dtype=torch.float32)
+    wt = torch.randn((n_out, in_features), generator=g, dtype=torch.float32) / in_features ** 0.5
+    bias = torch.randn((n_out,), generator=g, dtype=torch.float32) * 0.1
+    return x.to(torch.bfloat16), wt.to(torch.bfloat16), bias
+
+
 def all_states(w: Workload, inp: Inputs) -> dict:
     """{(seq, chunk, level): (K_raw, V_raw)} for prefilled states and nodes' own states."""
     st = dict(inp.history)
