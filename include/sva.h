@@ -198,6 +198,25 @@ sva_status sva_rope_kv_write_qknorm(sva_cache* c, const sva_node* nodes, int32_t
                                     const float* gamma_k, const float* gamma_q, float eps,
                                     sva_stream s);
 
+/* The linear projection in front of the attention layer, producing the
+ * token-major inputs of sva_rope_kv_write (the paper's denoiser is a DiT
+ * whose attention layers take q, k, v from the token features; Section 3.2
+ * reads K and V from them; the layer itself is not spelled out):
+ *   [q | k | v] = x W^T + b,  q, k, v each [rows][H*d] = [rows][H][d],
+ * with H, d from the cache's geometry.  bf16 operands, fp32 accumulation on
+ * the tensor cores, bias added in fp32, one bf16 rounding per output.
+ *   x       [rows][in_features] bf16 (e.g. rows = n_nodes * T token features)
+ *   weight  [3*H*d][in_features] bf16, out_features x in_features: q's output
+ *           rows first, then k's, then v's
+ *   bias    [3*H*d] fp32, or NULL
+ *   q, k, v [rows][H*d] bf16 outputs
+ * in_features a positive multiple of 8; H*d a multiple of 128; every pointer
+ * 16-byte aligned.  Stream-ordered; a device timeout is reported by
+ * sva_poll_device_status.  Errors: INVALID_ARGUMENT, UNSUPPORTED (H*d), CUDA. */
+sva_status sva_qkv_project(sva_cache* c, const void* x, int32_t rows, int32_t in_features,
+                           const void* weight, const float* bias, void* q, void* k, void* v,
+                           sva_stream s);
+
 /* Policy-indexed chunk-causal attention (Eq. 4) for a batch of nodes:
  *   out[i][u][h] = sum_v softmax_v(scale * q[i][u][h] . k_v + M(u, v)) v_v
  * over the keys of node i's own slot and its visible context slots; M is 0

@@ -17,7 +17,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libsva.so")
 
-SOURCES = ["attend.cu", "attend_noalloc.cu", "rope_kv.cu", "sva_api.cpp"]
+SOURCES = ["attend.cu", "attend_noalloc.cu", "rope_kv.cu", "qkv_gemm.cu", "sva_api.cpp"]
 HEADERS = [os.path.join(CSRC, h) for h in ("internal.h", "ptx.cuh")] + [os.path.join(INCLUDE, "sva.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-lineinfo", "-O3", "-std=c++17", "-Xcompiler", "-fPIC",

@@ -82,6 +82,20 @@ struct RopeParams {
   RopeNode nodes[SVA_MAX_NODES];
 };
 
+// The QKV projection y = x W^T + b split into q, k, v (sva_qkv_project).
+struct ProjParams {
+  CUtensorMap tmap_x;  // x as 2D (C, rows), box (64, 128), 128B swizzle
+  CUtensorMap tmap_w;  // weight as 2D (C, 3N), box (64, BN), 128B swizzle
+  const float* bias;   // [3N] fp32, or null
+  void* out[3];        // q, k, v: bf16 [rows][N]
+  int* status;         // device status word
+  int32_t rows, C, N;  // N = H * d outputs per tensor
+  int32_t n_mtiles, n_ntiles, n_kblocks;
+  uint64_t timeout_ns;
+};
+
+cudaError_t launch_qkv_project(const ProjParams& p, int block_n, int grid, cudaStream_t s);
+
 // Size of the library-owned split scratch used by sva_attend_nodes_noalloc.
 constexpr size_t kStaticScratchBytes = (size_t)32 << 20;
 

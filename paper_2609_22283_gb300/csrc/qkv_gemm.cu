@@ -1,0 +1,269 @@
+// The linear projection in front of the attention layer: for every token row
+// of x, y = x W^T + b, split into the q, k and v tensors that
+// sva_rope_kv_write consumes (token-major [rows][H*d] each).  A dense
+// contraction, so it runs on the tensor cores:
+//
+//   bf16 x [rows][C] (A, K-major) times bf16 W [3N][C] (B, K-major) into an
+//   fp32 accumulator in TMEM, 128 x BN output tiles (BN = 256, or 128 when
+//   N = H*d is not a multiple of 256), 64-wide K blocks through a 4-stage
+//   TMA ring.
+//
+// Persistent CTAs (one per SM) walk the output tiles; two TMEM accumulators
+// let the epilogue of one tile (TMEM -> + bias -> bf16 -> global) overlap the
+// main loop of the next.
+//   warp 0     TMA producer (x and W tiles, 128-byte swizzle);
+//   warp 1     TMEM owner and MMA issuer (whole warp, one elected lane);
+//   warps 4-7  epilogue, one output row per thread.
+// A tile never straddles q, k and v (N is a multiple of BN), so its epilogue
+// writes into one tensor.  Rows past `rows` read zeros (TMA fill) and are
+// not stored; K past C reads zeros on both operands.  All waits are bounded:
+// on expiry the CTA records SVA_ERR_DEVICE_TIMEOUT, drains its own copies and
+// MMAs, frees TMEM and exits.
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace sva {
+namespace {
+
+using namespace ptx;
+
+constexpr int kProjThreads = 256;
+constexpr int kStages = 4;
+constexpr int kBM = 128;
+constexpr int kBK = 64;
+
+template <int BN>
+struct ProjCfg {
+  static constexpr int kABytes = kBM * kBK * 2;  // 16 KB
+  static constexpr int kBBytes = BN * kBK * 2;   // 32 KB at BN = 256
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024;  // + alignment slack
+  static constexpr uint32_t kTmemCols = 2 * BN;                   // two accumulators
+};
+
+struct ProjBars {
+  uint64_t full[kStages];
+  uint64_t empty[kStages];
+  uint64_t acc_full[2];
+  uint64_t acc_empty[2];
+  uint64_t drain;
+};
+
+__device__ __forceinline__ uint32_t pack2_bf16(float lo, float hi) {
+  __nv_bfloat162 r = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&r);
+}
+
+__device__ __forceinline__ void proj_timeout(const ProjParams& p, volatile int* abort_flag) {
+  *abort_flag = 1;
+  atomicCAS(p.status, kStatusOk, kStatusTimeout);
+}
+
+template <int BN>
+__global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __grid_constant__ ProjParams p) {
+  using C = ProjCfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  __shared__ ProjBars bars;
+  __shared__ uint32_t tmem_base_sh;
+  __shared__ volatile int abort_flag;
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int total = p.n_mtiles * p.n_ntiles;
+
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&bars.full[s], 1);
+      mbar_init(&bars.empty[s], 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&bars.acc_full[b], 1);
+      mbar_init(&bars.acc_empty[b], 128);
+    }
+    mbar_init(&bars.drain, 1);
+    fence_mbar_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(&tmem_base_sh, C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tbase = tmem_base_sh;
+  const uint64_t tmo = p.timeout_ns;
+  int issued = 0;  // producer: K blocks whose copies were started
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      prefetch_tmap(&p.tmap_x);
+      prefetch_tmap(&p.tmap_w);
+      bool ok = true;
+      for (int t = blockIdx.x; ok && t < total; t += gridDim.x) {
+        const int m = t / p.n_ntiles, n = t - (t / p.n_ntiles) * p.n_ntiles;
+        for (int kb = 0; kb < p.n_kblocks; ++kb, ++issued) {
+          const int s = issued % kStages;
+          const uint32_t ph = (uint32_t)(issued / kStages) & 1u;
+          if (!mbar_wait(&bars.empty[s], ph ^ 1u, &abort_flag, tmo)) {
+            proj_timeout(p, &abort_flag);
+            ok = false;
+            break;
+          }
+          uint8_t* sa = smem + s * C::kStageBytes;
+          mbar_arrive_expect_tx(&bars.full[s], C::kStageBytes);
+          tma_load_2d(sa, &p.tmap_x, &bars.full[s], kb * kBK, m * kBM);
+          tma_load_2d(sa + C::kABytes, &p.tmap_w, &bars.full[s], kb * kBK, n * BN);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    constexpr uint32_t idesc = idesc_bf16_f32(kBM, BN, false);
+    const uint64_t dA = sdesc_sw128(smem_u32(smem), 16, 1024);
+    const uint64_t dB = sdesc_sw128(smem_u32(smem + C::kABytes), 16, 1024);
+    constexpr uint64_t kStageStep = (uint64_t)(C::kStageBytes >> 4);
+    auto wait = [&](uint64_t* bar, uint32_t parity) {
+      return __all_sync(0xffffffffu, mbar_wait(bar, parity, &abort_flag, tmo));
+    };
+    bool ok = true;
+    int it = 0, tc = 0;
+    for (int t = blockIdx.x; ok && t < total; t += gridDim.x, ++tc) {
+      const int acc = tc & 1;
+      if (!wait(&bars.acc_empty[acc], ((uint32_t)(tc >> 1) & 1u) ^ 1u)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const uint32_t dcol = tbase + (uint32_t)(acc * BN);
+      for (int kb = 0; kb < p.n_kblocks; ++kb, ++it) {
+        const int s = it % kStages;
+        if (!wait(&bars.full[s], (uint32_t)(it / kStages) & 1u)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint64_t a = dA + (uint64_t)s * kStageStep;
+        const uint64_t b = dB + (uint64_t)s * kStageStep;
+#pragma unroll
+        for (int kk = 0; kk < kBK / 16; ++kk)  // 32 bytes of K per MMA inside the swizzle atom
+          mma_ss_warp(dcol, a + (uint64_t)(kk * 2), b + (uint64_t)(kk * 2), idesc,
+                      (kb > 0 || kk > 0) ? 1u : 0u);
+        mma_commit_warp(&bars.empty[s]);  // the stage is free once these MMAs have read it
+      }
+      if (!ok) break;
+      mma_commit_warp(&bars.acc_full[acc]);
+    }
+    if (!ok && lane == 0) proj_timeout(p, &abort_flag);
+  } else if (warp >= 4) {
+    // ------------------------------------------------------------ epilogue
+    const int q4 = warp & 3;
+    const int row = q4 * 32 + lane;
+    const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
+    bool ok = true;
+    int tc = 0;
+    for (int t = blockIdx.x; ok && t < total; t += gridDim.x, ++tc) {
+      const int m = t / p.n_ntiles, n = t - (t / p.n_ntiles) * p.n_ntiles;
+      const int acc = tc & 1;
+      ok = mbar_wait(&bars.acc_full[acc], (uint32_t)(tc >> 1) & 1u, &abort_flag, tmo);
+      ok = __all_sync(0xffffffffu, ok);
+      if (!ok) break;
+      tc_fence_after();
+      const int col = n * BN;            // output column in [0, 3N)
+      const int tensor = col / p.N;      // q, k or v
+      const int c0 = col - tensor * p.N;  // column inside that tensor
+      const long long grow = (long long)m * kBM + row;
+      const bool in_range = grow < p.rows;
+      __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.out[tensor]) + grow * p.N + c0;
+#pragma unroll 1
+      for (int c = 0; c < BN / 32; ++c) {
+        uint32_t r[32];
+        tmem_ld32(tbase + lane_off + (uint32_t)(acc * BN + c * 32), r);
+        tmem_wait_ld(r);
+        float bv[32];
+        if (p.bias != nullptr) {
+          const float4* b4 = reinterpret_cast<const float4*>(p.bias + col + c * 32);
+#pragma unroll
+          for (int v = 0; v < 8; ++v) {
+            const float4 x = __ldg(b4 + v);
+            bv[4 * v] = x.x; bv[4 * v + 1] = x.y; bv[4 * v + 2] = x.z; bv[4 * v + 3] = x.w;
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < 32; ++e) bv[e] = 0.0f;
+        }
+        if (in_range) {
+          uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
+#pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            uint4 w;
+            w.x = pack2_bf16(__uint_as_float(r[8 * v + 0]) + bv[8 * v + 0], __uint_as_float(r[8 * v + 1]) + bv[8 * v + 1]);
+            w.y = pack2_bf16(__uint_as_float(r[8 * v + 2]) + bv[8 * v + 2], __uint_as_float(r[8 * v + 3]) + bv[8 * v + 3]);
+            w.z = pack2_bf16(__uint_as_float(r[8 * v + 4]) + bv[8 * v + 4], __uint_as_float(r[8 * v + 5]) + bv[8 * v + 5]);
+            w.w = pack2_bf16(__uint_as_float(r[8 * v + 6]) + bv[8 * v + 6], __uint_as_float(r[8 * v + 7]) + bv[8 * v + 7]);
+            d4[v] = w;
+          }
+        }
+      }
+      tc_fence_before();
+      mbar_arrive(&bars.acc_empty[acc]);  // the MMA warp may overwrite this accumulator
+    }
+    if (!ok) proj_timeout(p, &abort_flag);
+  }
+
+  // ---------------------------------------------------------------- teardown
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (abort_flag) {
+    // Some wait expired: wait (bounded, ignoring the abort flag) for the
+    // copies this CTA started and for every MMA it issued before exiting.
+    const int zero = 0;
+    if (warp == 0 && lane == 0) {
+      for (int i = (issued > kStages ? issued - kStages : 0); i < issued; ++i)
+        mbar_wait(&bars.full[i % kStages], (uint32_t)(i / kStages) & 1u, &zero, tmo);
+    } else if (warp == 1) {
+      mma_commit_warp(&bars.drain);
+      mbar_wait(&bars.drain, 0, &zero, tmo);
+    }
+  }
+  __syncwarp();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tbase, C::kTmemCols);
+  }
+}
+
+template <int BN>
+cudaError_t launch_bn(const ProjParams& p, int grid, cudaStream_t s) {
+  using C = ProjCfg<BN>;
+  static bool configured[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (!configured[dev]) {
+    e = cudaFuncSetAttribute(qkv_project_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             C::kSmemBytes);
+    if (e != cudaSuccess) return e;
+    configured[dev] = true;
+  }
+  qkv_project_kernel<BN><<<grid, kProjThreads, C::kSmemBytes, s>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_qkv_project(const ProjParams& p, int block_n, int grid, cudaStream_t s) {
+  if (block_n == 256) return launch_bn<256>(p, grid, s);
+  if (block_n == 128) return launch_bn<128>(p, grid, s);
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace sva

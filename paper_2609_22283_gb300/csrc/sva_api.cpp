@@ -683,6 +683,70 @@ sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes
   return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, s);
 }
 
+sva_status sva_qkv_project(sva_cache* c, const void* x, int32_t rows, int32_t in_features,
+                           const void* weight, const float* bias, void* q, void* k, void* v,
+                           sva_stream s) {
+  if (c == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "NULL cache");
+  if (rows < 1 || in_features < 8 || in_features % 8 != 0)
+    return fail(SVA_ERR_INVALID_ARGUMENT,
+                "rows %d must be >= 1 and in_features %d a positive multiple of 8", rows,
+                in_features);
+  if (x == nullptr || weight == nullptr || q == nullptr || k == nullptr || v == nullptr ||
+      !aligned16(x) || !aligned16(weight) || !aligned16(q) || !aligned16(k) || !aligned16(v) ||
+      (bias != nullptr && !aligned16(bias)))
+    return fail(SVA_ERR_INVALID_ARGUMENT,
+                "x, weight, q, k, v (and bias if given) must be non-NULL and 16-byte aligned");
+  sva_status st = check_device(c);
+  if (st != SVA_OK) return st;
+  const sva_geometry& g = c->g;
+  const int N = g.num_heads * g.head_dim;
+  if (N % 128 != 0)
+    return fail(SVA_ERR_UNSUPPORTED, "num_heads * head_dim = %d is not a multiple of 128", N);
+  const int bn = (N % 256 == 0) ? 256 : 128;
+  auto fn = encode_fn();
+  if (!fn) return fail(SVA_ERR_CUDA, "cuTensorMapEncodeTiled is not available from the driver");
+  static thread_local sva::ProjParams p;
+  std::memset(&p, 0, sizeof(p));
+  cuuint32_t es[2] = {1, 1};
+  {
+    cuuint64_t dims[2] = {(cuuint64_t)in_features, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)in_features * 2};
+    cuuint32_t box[2] = {64, 128};
+    CUresult r = fn(&p.tmap_x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(x), dims,
+                    strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(SVA_ERR_CUDA, "cuTensorMapEncodeTiled(x) failed: %d", (int)r);
+  }
+  {
+    cuuint64_t dims[2] = {(cuuint64_t)in_features, (cuuint64_t)3 * N};
+    cuuint64_t strides[1] = {(cuuint64_t)in_features * 2};
+    cuuint32_t box[2] = {64, (cuuint32_t)bn};
+    CUresult r = fn(&p.tmap_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(weight),
+                    dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+      return fail(SVA_ERR_CUDA, "cuTensorMapEncodeTiled(weight) failed: %d", (int)r);
+  }
+  p.bias = bias;
+  p.out[0] = q;
+  p.out[1] = k;
+  p.out[2] = v;
+  p.status = reinterpret_cast<int*>(c->base + c->L.status);
+  p.rows = rows;
+  p.C = in_features;
+  p.N = N;
+  p.n_mtiles = (rows + 127) / 128;
+  p.n_ntiles = 3 * N / bn;
+  p.n_kblocks = (in_features + 63) / 64;
+  p.timeout_ns = c->timeout_ns;
+  const long long tiles = (long long)p.n_mtiles * p.n_ntiles;
+  const int grid = (int)std::min<long long>(tiles, c->num_sms);
+  cudaError_t e = sva::launch_qkv_project(p, bn, grid, reinterpret_cast<cudaStream_t>(s));
+  if (e != cudaSuccess) return cuda_fail(e, "qkv_project launch");
+  return ok();
+}
+
 sva_status sva_attend_nodes_sparse(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
                                    const void* q, void* out, float* lse, float scale,
                                    const uint32_t* tile_mask, int32_t words_per_row,

@@ -38,7 +38,7 @@ MAX_NODES = 64
 EXPORTED = ("sva_cache_bytes", "sva_cache_create", "sva_cache_bind", "sva_cache_lookup",
             "sva_cache_release", "sva_select_context", "sva_pipeline_round", "sva_check_pipeline",
             "sva_rope_kv_write", "sva_rope_kv_write_qknorm", "sva_attend_nodes",
-            "sva_attend_nodes_sparse", "sva_attend_workspace_bytes",
+            "sva_attend_nodes_sparse", "sva_qkv_project", "sva_attend_workspace_bytes",
             "sva_cache_set_workspace", "sva_attend_nodes_noalloc", "sva_poll_device_status",
             "sva_debug_inject", "sva_destroy", "sva_last_error")
 
@@ -91,6 +91,7 @@ def load(path: str = LIB_PATH):
         "sva_rope_kv_write_qknorm": ([p, pn, i32, p, p, p, p, p, ctypes.c_float, p], i32),
         "sva_attend_nodes": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
         "sva_attend_nodes_sparse": ([p, pn, i32, p, p, p, ctypes.c_float, p, i32, p], i32),
+        "sva_qkv_project": ([p, p, i32, i32, p, p, p, p, p, p], i32),
         "sva_attend_workspace_bytes": ([p], ctypes.c_size_t),
         "sva_attend_nodes_noalloc": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
         "sva_cache_set_workspace": ([p, p, ctypes.c_size_t], i32),
@@ -310,6 +311,35 @@ class Cache:
                                           float(scale), ctypes.c_void_p(tile_mask.data_ptr()),
                                           int(tile_mask.shape[2]),
                                           ctypes.c_void_p(_stream_handle(stream)))
+        _check(st)
+
+    def qkv_project(self, x, weight, bias, q, k, v, stream=None, check=True):
+        """sva_qkv_project: [q | k | v] = x W^T + b.  x [..., C] bf16 (rows = all
+        leading dims), weight [3*H*d][C] bf16, bias [3*H*d] fp32 or None, q, k, v
+        bf16 with rows * H * d elements each (e.g. [n][T][H][d]); all contiguous
+        CUDA tensors."""
+        g = self.g
+        n_out = g.num_heads * g.head_dim
+        C = int(x.shape[-1])
+        rows = x.numel() // C
+        if check:
+            for t, nm in ((x, "x"), (weight, "weight"), (q, "q"), (k, "k"), (v, "v")):
+                if t.dtype != torch.bfloat16 or not t.is_cuda or not t.is_contiguous():
+                    raise ValueError(f"{nm} must be a contiguous bf16 CUDA tensor")
+            if tuple(weight.shape) != (3 * n_out, C):
+                raise ValueError(f"weight must be [{3 * n_out}][{C}]")
+            for t, nm in ((q, "q"), (k, "k"), (v, "v")):
+                if t.numel() != rows * n_out:
+                    raise ValueError(f"{nm} must hold rows * H * d = {rows * n_out} elements")
+            if bias is not None and (bias.dtype != torch.float32 or not bias.is_cuda
+                                     or not bias.is_contiguous() or bias.numel() != 3 * n_out):
+                raise ValueError(f"bias must be a contiguous fp32 CUDA tensor of {3 * n_out}")
+        st = _lib.sva_qkv_project(self.handle, ctypes.c_void_p(x.data_ptr()), rows, C,
+                                  ctypes.c_void_p(weight.data_ptr()),
+                                  ctypes.c_void_p(bias.data_ptr() if bias is not None else 0),
+                                  ctypes.c_void_p(q.data_ptr()), ctypes.c_void_p(k.data_ptr()),
+                                  ctypes.c_void_p(v.data_ptr()),
+                                  ctypes.c_void_p(_stream_handle(stream)))
         _check(st)
 
     def workspace_bytes(self) -> int:

@@ -1,0 +1,108 @@
+"""GPU parity of the QKV projection (sva_qkv_project, the tcgen05 GEMM that
+feeds sva_rope_kv_write) against the fp64 oracle, and of the chain
+projection -> RoPE + cache write -> attention against the oracle's chain.
+
+Tolerance (derived from the arithmetic): the library rounds each fp32
+accumulator to bf16 once (at most 2^-9 relative) and accumulates in fp32 in
+its own order; element bound |d| <= 2^-8 |y| + 1e-3 rms(y), and a relative
+RMS of 2e-3."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2609_22283_gb300 import inputs as I
+from paper_2609_22283_gb300 import sva
+from paper_2609_22283_gb300.pipeline import Step, geometry_for
+from tests import _parity as P
+
+pytestmark = pytest.mark.gpu
+
+
+def _check(got, ref, what):
+    got = got.astype(np.float64)
+    rms = float(np.sqrt(np.mean(ref ** 2)))
+    bound = 2.0 ** -8 * np.abs(ref) + 1e-3 * rms
+    bad = np.abs(got - ref) > bound
+    assert not bad.any(), f"{what}: {int(bad.sum())} elements out of bound, max |d| {np.abs(got - ref).max():.3e}"
+    rr = float(np.linalg.norm(got - ref) / np.linalg.norm(ref))
+    assert rr <= 2e-3, f"{what}: rel rms {rr:.3e}"
+
+
+def _project(w, C, rows_sample=None, bias=True):
+    x, wt, b = I.projection_inputs(w, C)
+    cache = sva.Cache(geometry_for(w))
+    dev = torch.device("cuda")
+    xd, wd = x.to(dev).contiguous(), wt.to(dev).contiguous()
+    bd = b.to(dev) if bias else None
+    outs = [torch.empty((w.n_nodes, w.T, w.H, w.d), dtype=torch.bfloat16, device=dev) for _ in range(3)]
+    cache.qkv_project(xd, wd, bd, *outs)
+    assert cache.poll() == 0
+    got = [o.float().cpu().numpy().reshape(-1, w.H, w.d) for o in outs]
+    xs = x.double().numpy().reshape(-1, C)
+    idx = np.arange(xs.shape[0]) if rows_sample is None else np.asarray(rows_sample)
+    ref = oracle.qkv_project(xs[idx], wt.double().numpy(), b.double().numpy() if bias else None, heads=w.H)
+    for t in range(3):
+        _check(got[t][idx], ref[t], f"{w.name} C={C} tensor {'qkv'[t]}")
+    cache.close()
+
+
+@pytest.mark.parametrize("C", [192, 200])
+def test_tiny_projection_all_rows(oracle_mod, C):
+    _project(I.WORKLOADS["tiny"], C)          # H*d = 128: 128-wide tiles; C = 200: ragged K block
+
+
+def test_tinys_projection_no_bias(oracle_mod):
+    _project(I.WORKLOADS["tinys"], 256, bias=False)
+
+
+def test_wan_geometry_projection_sampled(oracle_mod):
+    # 4 x 4680 token rows (ragged last 128-row tile), 1536 -> 3 x 12 x 128
+    w = I.WORKLOADS["prog4"]
+    rng = np.random.default_rng(21)
+    rows = sorted(set(rng.choice(w.n_nodes * w.T, 300, replace=False).tolist()) | {0, 18719, 18688, 127, 128})
+    _project(w, 1536, rows)
+
+
+def test_projection_feeds_rope_and_attention(oracle_mod):
+    """x -> sva_qkv_project -> sva_rope_kv_write -> sva_attend_nodes against the
+    oracle's projection (rounded to bf16 as stored) -> node_forward."""
+    w = I.WORKLOADS["tiny"]
+    C = 128
+    inp = I.generate(w)                        # history states stay the seeded ones
+    x, wt, b = I.projection_inputs(w, C)
+    dev = torch.device("cuda")
+    step = Step(w)
+    step.prefill(inp)
+    q, k, v = (torch.empty((w.n_nodes, w.T, w.H, w.d), dtype=torch.bfloat16, device=dev) for _ in range(3))
+    step.cache.qkv_project(x.to(dev).contiguous(), wt.to(dev).contiguous(), b.to(dev), q, k, v)
+    out, lse = step.outputs()
+    step.run(q, k, v, out, lse)
+    assert step.cache.poll() == 0
+    rq, rk, rv = oracle.qkv_project(x.double().numpy().reshape(-1, C), wt.double().numpy(),
+                                    b.double().numpy(), heads=w.H)
+    shape = (w.n_nodes, w.T, w.H, w.d)
+    rq, rk, rv = (torch.from_numpy(oracle.bf16(t).reshape(shape)) for t in (rq, rk, rv))
+    inp2 = I.Inputs(inp.history, rq, rk, rv)
+    states = P.oracle_states(w, inp2)
+    got = out.float().cpu().numpy()
+    for i in range(w.n_nodes):
+        ref, _ = P.oracle_node(w, inp2, states, i, range(w.H), range(w.T))
+        for h in range(w.H):
+            P.assert_close(got[i, :, h, :], ref[h], f"projection chain node {i} head {h}")
+    step.close()
+
+
+def test_projection_argument_errors(sva_mod):
+    w = I.WORKLOADS["tiny"]
+    cache = sva.Cache(geometry_for(w))
+    lib = sva_mod.load()
+    z = torch.zeros(64 * 128, dtype=torch.bfloat16, device="cuda")
+    p = lambda t: __import__("ctypes").c_void_p(t.data_ptr())
+    st = lib.sva_qkv_project(cache.handle, p(z), 64, 100, p(z), None, p(z), p(z), p(z), None)
+    assert st == sva_mod.ERR_INVALID_ARGUMENT      # in_features not a multiple of 8
+    st = lib.sva_qkv_project(cache.handle, None, 64, 128, p(z), None, p(z), p(z), p(z), None)
+    assert st == sva_mod.ERR_INVALID_ARGUMENT
+    cache.close()
