@@ -465,6 +465,8 @@ def run_ours(args, world, rank, local):
     }
     if remeasured:
         line["clocks_note"] = "first timed region saw a slowdown reason; re-measured once"
+    if not args.no_projection:
+        line["qkv_project"] = time_projection(step, w, dev, flush, stream, peak, world)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         tf, rows, secs, cores = oracle_sample(w, inp, args.cpu_seconds)
         line["cpu_baseline"] = {
@@ -475,6 +477,38 @@ def run_ours(args, world, rank, local):
         print(json.dumps(line), flush=True)
     step.close()
     return 0
+
+
+def time_projection(step, w, dev, flush, stream, peak, world):
+    """The input projection in front of the step (sva_qkv_project: [q | k | v] =
+    x W^T + b for the step's n*T token rows, hidden size H*d), timed like the
+    step: CUDA events per launch, L2 flushed between launches.  Reported
+    beside the step, not inside it."""
+    import torch
+    from paper_2609_22283_gb300 import inputs as I
+    C = w.H * w.d
+    x, wt, b = I.projection_inputs(w, C)
+    x, wt, b = x.to(dev), wt.to(dev), b.to(dev)
+    outs = [torch.empty((w.n_nodes, w.T, w.H, w.d), dtype=torch.bfloat16, device=dev) for _ in range(3)]
+    for _ in range(3):
+        step.cache.qkv_project(x, wt, b, *outs, check=False)
+    K = 20
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
+    torch.cuda.synchronize()
+    for e0, e1 in ev:
+        flush.zero_()
+        e0.record(stream)
+        step.cache.qkv_project(x, wt, b, *outs, check=False)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    if step.cache.poll() != 0:
+        raise RuntimeError("device status after the projection")
+    ms = reduce_max(sum(a.elapsed_time(c) for a, c in ev) / K, world)
+    flops = 2.0 * w.n_nodes * w.T * C * 3 * C
+    tf = flops / (ms * 1e-3) / 1e12
+    return {"kernel": "qkv_project_kernel", "rows": w.n_nodes * w.T, "in_features": C,
+            "out_features": 3 * C, "ms": ms, "achieved": tf, "unit": "TFLOP/s",
+            "peak": peak, "frac": tf / peak, "launches": K}
 
 
 def compare_schedules(args):
@@ -552,6 +586,8 @@ def main():
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--reference-seconds", type=float, default=8.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-projection", action="store_true",
+                    help="skip timing the QKV projection beside the step")
     ap.add_argument("--compare-schedules", action="store_true",
                     help="time clean-serial against progressive-pipeline execution of one chunk")
     args = ap.parse_args()
