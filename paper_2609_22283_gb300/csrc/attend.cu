@@ -536,7 +536,10 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         tmem_wait_ld(s[1]);
         tmem_wait_ld_max2(cmax);
         float m_part = fmaxf(cmax[0], cmax[1]);
-        if (__any_sync(0xffffffffu, vrel < 64)) {
+        // Tiles that can hold masked keys (a slot's ragged last tile, the own
+        // chunk under frame causality) take the masked path; the test is the
+        // same for every thread, so it needs no vote.
+        if (valid_tile < kTile || own_fc) {
           float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
           for (int c = 0; c < 2; ++c)
