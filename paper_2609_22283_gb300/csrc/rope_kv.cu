@@ -125,43 +125,58 @@ __global__ void __launch_bounds__(256) rope_kv_kernel(const __grid_constant__ Ro
       rk = __frsqrt_rn(__fmaf_rn(sk, inv_n, p.norm_eps));
       rq = __frsqrt_rn(__fmaf_rn(sq, inv_n, p.norm_eps));
     }
-#pragma unroll 4
-    for (int v = lane; v < per_tok; v += 32) {
-      const int h = v >> vshift;
-      const size_t in_off = in_tok + (size_t)v * 8;
-      const uint4 kv = ld_stream(kin + in_off);
-      const uint4 vv = ld_stream(vin + in_off);
-      uint4 qv = make_uint4(0, 0, 0, 0);
-      if (qio) qv = *reinterpret_cast<const uint4*>(qio + in_off);
-      uint32_t kw[4] = {kv.x, kv.y, kv.z, kv.w};
-      uint32_t qw[4] = {qv.x, qv.y, qv.z, qv.w};
-      if (norm) {
-        const float4* gk = reinterpret_cast<const float4*>(p.gamma_k + (size_t)v * 8);
-        const float4 gk0 = __ldg(gk), gk1 = __ldg(gk + 1);
-        const float gkk[8] = {gk0.x, gk0.y, gk0.z, gk0.w, gk1.x, gk1.y, gk1.z, gk1.w};
+    // Batches of kBatch vectors per lane: every load of a batch is issued
+    // before any of its stores (q is rotated in place, so without the split
+    // the compiler keeps each iteration's loads behind the previous stores).
+    constexpr int kBatch = 4;
+    for (int v0 = lane; v0 < per_tok; v0 += 32 * kBatch) {
+      uint4 kv[kBatch], vv[kBatch], qv[kBatch];
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-          kw[k] = norm_rotate_pair(kw[k], gkk[2 * k] * rk, gkk[2 * k + 1] * rk, cs[k].x, cs[k].y);
-        if (qio) {
-          const float4* gq = reinterpret_cast<const float4*>(p.gamma_q + (size_t)v * 8);
-          const float4 gq0 = __ldg(gq), gq1 = __ldg(gq + 1);
-          const float gqq[8] = {gq0.x, gq0.y, gq0.z, gq0.w, gq1.x, gq1.y, gq1.z, gq1.w};
-#pragma unroll
-          for (int k = 0; k < 4; ++k)
-            qw[k] = norm_rotate_pair(qw[k], gqq[2 * k] * rq, gqq[2 * k + 1] * rq, cs[k].x,
-                                     cs[k].y);
-        }
-      } else {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          kw[k] = rotate_pair(kw[k], cs[k].x, cs[k].y);
-          qw[k] = rotate_pair(qw[k], cs[k].x, cs[k].y);
+      for (int j = 0; j < kBatch; ++j) {
+        const int v = v0 + 32 * j;
+        if (v < per_tok) {
+          const size_t in_off = in_tok + (size_t)v * 8;
+          kv[j] = ld_stream(kin + in_off);
+          vv[j] = ld_stream(vin + in_off);
+          qv[j] = qio ? *reinterpret_cast<const uint4*>(qio + in_off) : make_uint4(0, 0, 0, 0);
         }
       }
-      __nv_bfloat16* kdst = cache + ((out_slot + (size_t)h * p.Tpad + u) * p.d + c8 * 8);
-      *reinterpret_cast<uint4*>(kdst) = make_uint4(kw[0], kw[1], kw[2], kw[3]);
-      *reinterpret_cast<uint4*>(kdst + kv_stride) = vv;
-      if (qio) *reinterpret_cast<uint4*>(qio + in_off) = make_uint4(qw[0], qw[1], qw[2], qw[3]);
+#pragma unroll
+      for (int j = 0; j < kBatch; ++j) {
+        const int v = v0 + 32 * j;
+        if (v >= per_tok) break;
+        const int h = v >> vshift;
+        const size_t in_off = in_tok + (size_t)v * 8;
+        uint32_t kw[4] = {kv[j].x, kv[j].y, kv[j].z, kv[j].w};
+        uint32_t qw[4] = {qv[j].x, qv[j].y, qv[j].z, qv[j].w};
+        if (norm) {
+          const float4* gk = reinterpret_cast<const float4*>(p.gamma_k + (size_t)v * 8);
+          const float4 gk0 = __ldg(gk), gk1 = __ldg(gk + 1);
+          const float gkk[8] = {gk0.x, gk0.y, gk0.z, gk0.w, gk1.x, gk1.y, gk1.z, gk1.w};
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            kw[k] = norm_rotate_pair(kw[k], gkk[2 * k] * rk, gkk[2 * k + 1] * rk, cs[k].x, cs[k].y);
+          if (qio) {
+            const float4* gq = reinterpret_cast<const float4*>(p.gamma_q + (size_t)v * 8);
+            const float4 gq0 = __ldg(gq), gq1 = __ldg(gq + 1);
+            const float gqq[8] = {gq0.x, gq0.y, gq0.z, gq0.w, gq1.x, gq1.y, gq1.z, gq1.w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k)
+              qw[k] = norm_rotate_pair(qw[k], gqq[2 * k] * rq, gqq[2 * k + 1] * rq, cs[k].x,
+                                       cs[k].y);
+          }
+        } else {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            kw[k] = rotate_pair(kw[k], cs[k].x, cs[k].y);
+            qw[k] = rotate_pair(qw[k], cs[k].x, cs[k].y);
+          }
+        }
+        __nv_bfloat16* kdst = cache + ((out_slot + (size_t)h * p.Tpad + u) * p.d + c8 * 8);
+        *reinterpret_cast<uint4*>(kdst) = make_uint4(kw[0], kw[1], kw[2], kw[3]);
+        *reinterpret_cast<uint4*>(kdst + kv_stride) = vv[j];
+        if (qio) *reinterpret_cast<uint4*>(qio + in_off) = make_uint4(qw[0], qw[1], qw[2], qw[3]);
+      }
     }
   }
 }
