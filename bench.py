@@ -467,6 +467,10 @@ def run_ours(args, world, rank, local):
         line["clocks_note"] = "first timed region saw a slowdown reason; re-measured once"
     if not args.no_projection:
         line["qkv_project"] = time_projection(step, w, dev, flush, stream, peak, world)
+        # the attention layer's three device steps: projection, RoPE + cache
+        # write, attention (kernel times summed; the projection is not in `value`)
+        line["nodes_per_s_with_projection"] = (
+            w.n_nodes * world / ((line["qkv_project"]["ms"] + t_step_ms) * 1e-3))
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         tf, rows, secs, cores = oracle_sample(w, inp, args.cpu_seconds)
         line["cpu_baseline"] = {
