@@ -1,0 +1,29 @@
+"""bench.py's algorithmic FLOP counts (CPU): the dense count is 4*T*Lkv*d*H
+per node written out from the workload's geometry, and the block-sparse
+count keeps only the mask's (query tile, key tile) pairs: an all-ones mask
+gives the dense count, the own-chunk-only mask gives a node without history."""
+import os
+import sys
+
+sys.path.insert(0, os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+
+import bench  # noqa: E402
+from paper_2609_22283_gb300 import inputs as I  # noqa: E402
+
+
+def test_dense_counts():
+    w = I.WORKLOADS["clean1"]
+    assert bench.attn_flops(w) == 4.0 * 4680 * (4 * 4680) * 128 * 12
+    w = I.WORKLOADS["prog4"]
+    assert bench.attn_flops(w) == 4 * 4.0 * 4680 * (7 * 4680) * 128 * 12
+
+
+def test_sparse_counts():
+    dense = I.WORKLOADS["tinys"]
+    ones = I.Workload(**{**dense.__dict__, "sparse": 1.0})
+    none = I.Workload(**{**dense.__dict__, "sparse": 0.0})
+    base = I.Workload(**{**dense.__dict__, "sparse": None})
+    assert bench.attn_flops(ones) == bench.attn_flops(base)
+    own_only = sum(4.0 * dense.T * dense.T * dense.d * dense.H for _ in dense.nodes)
+    assert bench.attn_flops(none) == own_only
+    assert own_only < bench.attn_flops(dense) < bench.attn_flops(base)
