@@ -176,10 +176,14 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
-  // Work unit, head-major so the CTAs that share a head's K/V run together;
-  // the splits of a unit are adjacent.
-  const int split = blockIdx.x % p.n_split;
-  const int unit = blockIdx.x / p.n_split;
+  // Work unit, head-major so the CTAs that share a head's K/V run together.
+  // The first n_full units run unsplit (one CTA each, the full waves); the
+  // others are split n_split ways, the splits of a unit adjacent.
+  const bool whole = (int)blockIdx.x < p.n_full;
+  const int ns = whole ? 1 : p.n_split;  // key ranges of this unit
+  const int split = whole ? 0 : (int)(blockIdx.x - p.n_full) % p.n_split;
+  const int unit = whole ? (int)blockIdx.x : p.n_full + (int)(blockIdx.x - p.n_full) / p.n_split;
+  const int sunit = unit - p.n_full;     // index among the split units
   const int qp = unit % p.n_qp;
   const int rest = unit / p.n_qp;
   const int ni = rest % p.n_nodes;
@@ -192,8 +196,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
   // a block-sparse mask a contiguous range of the tiles either query tile
   // may attend (set in the prologue below).
   constexpr bool sparse = kSparse;  // a launch with a block-sparse tile mask
-  int t_begin = (int)((long long)split * n_all / p.n_split);
-  int n_tiles = (int)((long long)(split + 1) * n_all / p.n_split) - t_begin;
+  int t_begin = (int)((long long)split * n_all / ns);
+  int n_tiles = (int)((long long)(split + 1) * n_all / ns) - t_begin;
   // per query tile, bit i = kernel key tile i (block-sparse instances only)
   __shared__ uint32_t tmask[2][kSparse ? kMaskWords : 1];
   __shared__ int sp_first, sp_count;
@@ -247,8 +251,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       total += __popc(m0 | m1);
     }
     if (lane == 0) {
-      const int lo = (int)((long long)split * total / p.n_split);
-      const int hi = (int)((long long)(split + 1) * total / p.n_split);
+      const int lo = (int)((long long)split * total / ns);
+      const int hi = (int)((long long)(split + 1) * total / ns);
       int first = n_all, seen = 0;
       for (int w = 0; hi > lo && w < words; ++w) {
         uint32_t u = tmask[0][w] | tmask[1][w];
@@ -623,7 +627,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     float l_row[2];  // the row's whole sum: both halves, under the same max
 #pragma unroll
     for (int b = 0; b < 2; ++b) l_row[b] = l[b] + __shfl_xor_sync(0xffffffffu, l[b], 16);
-    if (p.n_split == 1) {
+    if (ns == 1) {
       if (ok) {
         tc_fence_after();
 #pragma unroll
@@ -666,7 +670,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       // Split unit.  Partial layout per (unit, split): O as [D/4][256]
       // float4 (rows of both query tiles), then m[256], then l[256].
       constexpr size_t kItem = (size_t)256 * (D + 2);
-      float* part = p.ws + ((size_t)unit * p.n_split + split) * kItem;
+      float* part = p.ws + ((size_t)sunit * ns + split) * kItem;
       if (ok) {
         tc_fence_after();
         float4* part4 = reinterpret_cast<float4*>(part);
@@ -703,13 +707,13 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       asm volatile("bar.sync 1, 256;" ::: "memory");
       if (threadIdx.x == 128) {
         int last = 0;
-        if (!abort_flag) last = atomicAdd(&p.ws_count[unit], 1) == p.n_split - 1;
+        if (!abort_flag) last = atomicAdd(&p.ws_count[sunit], 1) == ns - 1;
         last_split = last;
       }
       asm volatile("bar.sync 1, 256;" ::: "memory");
       if (last_split) {
         __threadfence();
-        const float* base = p.ws + (size_t)unit * p.n_split * kItem;
+        const float* base = p.ws + (size_t)sunit * ns * kItem;
 #pragma unroll
         for (int b = 0; b < 2; ++b) {
           if (b == 1 && !has_q1) break;
@@ -720,14 +724,14 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
           float M = -INFINITY;
 #pragma unroll
           for (int k = 0; k < kMaxSplit; ++k) {
-            mk[k] = k < p.n_split ? __ldcg(base + k * kItem + D * 256 + r) : -INFINITY;
+            mk[k] = k < ns ? __ldcg(base + k * kItem + D * 256 + r) : -INFINITY;
             M = fmaxf(M, mk[k]);
           }
           const float M_sub = (M == -INFINITY) ? 0.0f : M;  // every range empty: O = 0
           float L = 0.0f;
 #pragma unroll
           for (int k = 0; k < kMaxSplit; ++k) {
-            wk[k] = k < p.n_split
+            wk[k] = k < ns
                         ? __ldcg(base + k * kItem + D * 256 + 256 + r) * ex2(mk[k] - M_sub)
                         : 0.0f;
             L += wk[k];
@@ -746,8 +750,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
 #pragma unroll
             for (int k = 0; k < kMaxSplit; ++k) {
               const float4* b4 = reinterpret_cast<const float4*>(base + k * kItem);
-              x[k] = k < p.n_split ? __ldcg(b4 + (c8 * 2 + 0) * 256 + r) : make_float4(0.f, 0.f, 0.f, 0.f);
-              y[k] = k < p.n_split ? __ldcg(b4 + (c8 * 2 + 1) * 256 + r) : make_float4(0.f, 0.f, 0.f, 0.f);
+              x[k] = k < ns ? __ldcg(b4 + (c8 * 2 + 0) * 256 + r) : make_float4(0.f, 0.f, 0.f, 0.f);
+              y[k] = k < ns ? __ldcg(b4 + (c8 * 2 + 1) * 256 + r) : make_float4(0.f, 0.f, 0.f, 0.f);
             }
             float a[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
 #pragma unroll
@@ -765,7 +769,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
           if (p.lse != nullptr && half == 0)
             p.lse[((size_t)nd.q_index * p.H + h) * p.T + token] = (M + __log2f(L)) * 0.69314718055994531f;
         }
-        if (threadIdx.x == 128) p.ws_count[unit] = 0;  // ready for the next launch
+        if (threadIdx.x == 128) p.ws_count[sunit] = 0;  // ready for the next launch
       }
     }
     // ---------------------------------------------------------------- teardown (softmax)

@@ -49,7 +49,9 @@ struct alignas(128) AttnParams {
   int32_t valid_last;   // valid key rows in the last tile of a slot
   int32_t frame_tokens; // tokens per latent frame (Hp * Wp)
   int32_t fault_mode;   // 0 in production; see sva_api.cpp
-  int32_t n_split;      // key-range splits per work unit (1 = no split)
+  int32_t n_split;      // key-range splits per split work unit (1 = no split)
+  int32_t n_full;       // units 0..n_full-1 run unsplit (one CTA each); the
+                        // rest are split n_split ways (CTAs after them)
   float* ws;            // split partials [unit][split][(d + 2) * 256] fp32, or null
   int* ws_count;        // per-unit arrival counters, zero between launches, or null
   uint64_t timeout_ns;

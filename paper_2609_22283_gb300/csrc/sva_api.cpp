@@ -268,6 +268,29 @@ int choose_split(const sva_cache* c, long long units, int min_tiles) {
   return best_s;
 }
 
+// The split plan of a launch: units 0..n_full-1 unsplit, the rest split
+// n_split ways.  When the units fill some whole waves of one CTA per SM, those
+// waves run unsplit and only the partial last wave is split; that has the
+// makespan of splitting every unit (when it is no longer) with fewer CTAs,
+// fewer prologues and epilogues and fewer partials to merge.
+void plan_split(const sva_cache* c, long long units, int min_tiles, long long* n_full,
+                int* n_split) {
+  const long long sms = c->num_sms;
+  const int s_all = choose_split(c, units, min_tiles);
+  *n_full = 0;
+  *n_split = s_all;
+  if (s_all == 1 || units < sms) return;
+  const long long full = units / sms * sms, rest = units - full;
+  const int s_rest = choose_split(c, rest, min_tiles);
+  const double cost_all = (double)((units * s_all + sms - 1) / sms) / s_all;
+  const double cost_mixed =
+      (double)(full / sms) + (double)((rest * s_rest + sms - 1) / sms) / s_rest;
+  if (cost_mixed <= cost_all + 1e-9) {
+    *n_full = full;
+    *n_split = s_rest;
+  }
+}
+
 }  // namespace
 
 extern "C" {
@@ -663,12 +686,16 @@ sva_status attend(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const vo
   int min_tiles = 1 << 30;
   for (int i = 0; i < n_nodes; ++i) min_tiles = std::min(min_tiles, p.nodes[i].n_kv * p.nt_slot);
   const long long units = (long long)g.num_heads * n_nodes * p.n_qp;
-  p.n_split = choose_split(c, units, min_tiles);
+  long long n_full = 0;
+  int n_split = 1;
+  plan_split(c, units, min_tiles, &n_full, &n_split);
+  p.n_full = (int32_t)n_full;
+  p.n_split = n_split;
   if (p.n_split > 1) {
     p.ws_count = reinterpret_cast<int*>(c->ws);
     p.ws = reinterpret_cast<float*>(c->ws + ws_counter_bytes(c));
   }
-  const long long grid = units * p.n_split;
+  const long long grid = n_full + (units - n_full) * p.n_split;
   cudaError_t e = sva::launch_attend(p, g.head_dim, (int)grid, reinterpret_cast<cudaStream_t>(s));
   if (e != cudaSuccess) return cuda_fail(e, "attend launch");
   return ok();
