@@ -87,7 +87,7 @@ struct RopeParams {
 // The QKV projection y = x W^T + b split into q, k, v (sva_qkv_project).
 struct ProjParams {
   CUtensorMap tmap_x;  // x as 2D (C, rows), box (64, 128), 128B swizzle
-  CUtensorMap tmap_w;  // weight as 2D (C, 3N), box (64, BN), 128B swizzle
+  CUtensorMap tmap_w;  // weight as 2D (C, 3N), box (64, BN / 2), 128B swizzle
   const float* bias;   // [3N] fp32, or null
   void* out[3];        // q, k, v: bf16 [rows][N]
   int* status;         // device status word

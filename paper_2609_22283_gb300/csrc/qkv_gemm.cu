@@ -10,7 +10,11 @@
 //
 // Persistent CTAs (one per SM) walk the output tiles; two TMEM accumulators
 // let the epilogue of one tile (TMEM -> + bias -> bf16 -> global) overlap the
-// main loop of the next.
+// main loop of the next.  CTAs run in clusters of two that take vertically
+// adjacent tiles (same W rows): each loads its own x tile and half of the W
+// tile, multicast into both CTAs' shared memory, so a CTA pulls 32 KB per K
+// block from L2 instead of 48 KB (the 4-stage ring holds too little to hide
+// the L2 latency at 48 KB per 512 MMA cycles).
 //   warp 0     TMA producer (x and W tiles, 128-byte swizzle);
 //   warp 1     TMEM owner and MMA issuer (whole warp, one elected lane);
 //   warps 4-7  epilogue, one output row per thread.
@@ -46,7 +50,7 @@ struct ProjCfg {
 
 struct ProjBars {
   uint64_t full[kStages];
-  uint64_t empty[kStages];
+  uint64_t empty[kStages];  // both CTAs' MMAs have read the stage (two arrivals)
   uint64_t acc_full[2];
   uint64_t acc_empty[2];
   uint64_t drain;
@@ -55,6 +59,39 @@ struct ProjBars {
 __device__ __forceinline__ uint32_t pack2_bf16(float lo, float hi) {
   __nv_bfloat162 r = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&r);
+}
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// TMA 2D tile load written to the same offset of every CTA in `mask`, each
+// CTA's barrier at `bar`'s offset receiving the completed bytes.
+__device__ __forceinline__ void tma_load_2d_mc(void* dst, const CUtensorMap* map, uint64_t* bar,
+                                               int32_t c0, int32_t c1, uint16_t mask) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
+      " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "h"(mask)
+      : "memory");
+}
+
+// Arrives on the barrier at `bar`'s offset in every CTA of `mask` once this
+// thread's MMAs so far have completed (one elected lane of a converged warp).
+__device__ __forceinline__ void mma_commit_mc_warp(uint64_t* bar, uint16_t mask) {
+  asm volatile(
+      "{\n"
+      " .reg .pred e;\n"
+      " elect.sync _|e, 0xffffffff;\n"
+      " @e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n"
+      "}\n" ::"r"(smem_u32(bar)), "h"(mask)
+      : "memory");
 }
 
 __device__ __forceinline__ void proj_timeout(const ProjParams& p, volatile int* abort_flag) {
@@ -74,13 +111,18 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int total = p.n_mtiles * p.n_ntiles;
+  // pairs of tiles (m pair, n): cluster c takes pairs c, c + clusters, ...;
+  // CTA `rank` of the cluster computes m tile 2 * m_pair + rank
+  const uint32_t rank = cluster_rank();
+  const int cluster = blockIdx.x >> 1, clusters = gridDim.x >> 1;
+  const int n_mpairs = (p.n_mtiles + 1) >> 1;
+  const int total = n_mpairs * p.n_ntiles;
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&bars.full[s], 1);
-      mbar_init(&bars.empty[s], 1);
+      mbar_init(&bars.empty[s], 2);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bars.acc_full[b], 1);
@@ -95,6 +137,7 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
   }
   tc_fence_before();
   __syncthreads();
+  cluster_sync();  // both CTAs' barriers are initialised before either multicasts
   tc_fence_after();
   const uint32_t tbase = tmem_base_sh;
   const uint64_t tmo = p.timeout_ns;
@@ -106,8 +149,9 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
       prefetch_tmap(&p.tmap_x);
       prefetch_tmap(&p.tmap_w);
       bool ok = true;
-      for (int t = blockIdx.x; ok && t < total; t += gridDim.x) {
-        const int m = t / p.n_ntiles, n = t - (t / p.n_ntiles) * p.n_ntiles;
+      for (int t = cluster; ok && t < total; t += clusters) {
+        const int mp = t / p.n_ntiles, n = t - (t / p.n_ntiles) * p.n_ntiles;
+        const int m = 2 * mp + (int)rank;  // past the last m tile: rows read as zeros
         for (int kb = 0; kb < p.n_kblocks; ++kb, ++issued) {
           const int s = issued % kStages;
           const uint32_t ph = (uint32_t)(issued / kStages) & 1u;
@@ -119,7 +163,18 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
           uint8_t* sa = smem + s * C::kStageBytes;
           mbar_arrive_expect_tx(&bars.full[s], C::kStageBytes);
           tma_load_2d(sa, &p.tmap_x, &bars.full[s], kb * kBK, m * kBM);
-          tma_load_2d(sa + C::kABytes, &p.tmap_w, &bars.full[s], kb * kBK, n * BN);
+          // this CTA's half of the W tile, into both CTAs
+          tma_load_2d_mc(sa + C::kABytes + rank * (C::kBBytes / 2), &p.tmap_w, &bars.full[s],
+                         kb * kBK, n * BN + (int)rank * (BN / 2), 0x3);
+        }
+      }
+      // Every stage must be released by both CTAs' MMAs before this CTA may
+      // leave: the peer's commits arrive on this CTA's empty barriers.
+      for (int j = issued; ok && j < issued + kStages; ++j) {
+        if (!mbar_wait(&bars.empty[j % kStages], ((uint32_t)(j / kStages) & 1u) ^ 1u, &abort_flag,
+                       tmo)) {
+          proj_timeout(p, &abort_flag);
+          ok = false;
         }
       }
     }
@@ -134,7 +189,7 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
     };
     bool ok = true;
     int it = 0, tc = 0;
-    for (int t = blockIdx.x; ok && t < total; t += gridDim.x, ++tc) {
+    for (int t = cluster; ok && t < total; t += clusters, ++tc) {
       const int acc = tc & 1;
       if (!wait(&bars.acc_empty[acc], ((uint32_t)(tc >> 1) & 1u) ^ 1u)) {
         ok = false;
@@ -155,7 +210,9 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
         for (int kk = 0; kk < kBK / 16; ++kk)  // 32 bytes of K per MMA inside the swizzle atom
           mma_ss_warp(dcol, a + (uint64_t)(kk * 2), b + (uint64_t)(kk * 2), idesc,
                       (kb > 0 || kk > 0) ? 1u : 0u);
-        mma_commit_warp(&bars.empty[s]);  // the stage is free once these MMAs have read it
+        // the stage is free (in both CTAs: half of it came from the peer) once
+        // these MMAs have read it
+        mma_commit_mc_warp(&bars.empty[s], 0x3);
       }
       if (!ok) break;
       mma_commit_warp(&bars.acc_full[acc]);
@@ -168,8 +225,9 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
     bool ok = true;
     int tc = 0;
-    for (int t = blockIdx.x; ok && t < total; t += gridDim.x, ++tc) {
-      const int m = t / p.n_ntiles, n = t - (t / p.n_ntiles) * p.n_ntiles;
+    for (int t = cluster; ok && t < total; t += clusters, ++tc) {
+      const int mp = t / p.n_ntiles, n = t - (t / p.n_ntiles) * p.n_ntiles;
+      const int m = 2 * mp + (int)rank;
       const int acc = tc & 1;
       ok = mbar_wait(&bars.acc_full[acc], (uint32_t)(tc >> 1) & 1u, &abort_flag, tmo);
       ok = __all_sync(0xffffffffu, ok);
@@ -238,6 +296,7 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
     tc_fence_after();
     tmem_dealloc(tbase, C::kTmemCols);
   }
+  cluster_sync();  // neither CTA leaves while the other may still reach its shared memory
 }
 
 template <int BN>
@@ -254,7 +313,20 @@ cudaError_t launch_bn(const ProjParams& p, int grid, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
-  qkv_project_kernel<BN><<<grid, kProjThreads, C::kSmemBytes, s>>>(p);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)grid);
+  cfg.blockDim = dim3(kProjThreads);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, qkv_project_kernel<BN>, p);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

@@ -747,7 +747,7 @@ sva_status sva_qkv_project(sva_cache* c, const void* x, int32_t rows, int32_t in
   {
     cuuint64_t dims[2] = {(cuuint64_t)in_features, (cuuint64_t)3 * N};
     cuuint64_t strides[1] = {(cuuint64_t)in_features * 2};
-    cuuint32_t box[2] = {64, (cuuint32_t)bn};
+    cuuint32_t box[2] = {64, (cuuint32_t)bn / 2};  // each CTA of a pair loads half a W tile
     CUresult r = fn(&p.tmap_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(weight),
                     dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -767,8 +767,9 @@ sva_status sva_qkv_project(sva_cache* c, const void* x, int32_t rows, int32_t in
   p.n_ntiles = 3 * N / bn;
   p.n_kblocks = (in_features + 63) / 64;
   p.timeout_ns = c->timeout_ns;
-  const long long tiles = (long long)p.n_mtiles * p.n_ntiles;
-  const int grid = (int)std::min<long long>(tiles, c->num_sms);
+  // clusters of two CTAs, each cluster one (pair of m tiles, n tile) at a time
+  const long long pairs = (long long)((p.n_mtiles + 1) / 2) * p.n_ntiles;
+  const int grid = 2 * (int)std::min<long long>(pairs, c->num_sms / 2);
   cudaError_t e = sva::launch_qkv_project(p, bn, grid, reinterpret_cast<cudaStream_t>(s));
   if (e != cudaSuccess) return cuda_fail(e, "qkv_project launch");
   return ok();
