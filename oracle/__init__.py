@@ -221,7 +221,7 @@ def attend_rows(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float,
 def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
                  states: dict, q_raw: np.ndarray, heads, rows, scale: float,
                  hidden: frozenset = frozenset(), within: str = "bidirectional",
-                 norm=None, tile_mask=None):
+                 norm=None, tile_mask=None, own_mask=None):
     """One denoising node (seq, b, j), computed from raw (pre-RoPE) inputs.
 
     states: {(seq, chunk, level): (K_raw, V_raw)} with arrays [T][H][d] holding
@@ -240,6 +240,9 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
         query u (tile u // 128) sees key v of key state s (0 = own chunk,
         1 + j = j-th selected state) only if entry [u // 128][s * nt + v // 128]
         is true, nt = ceil(T / 128); a further mask on top of the others.
+    own_mask: None, or a boolean array [T][T] for the node: query u sees key v
+        of its own chunk only if own_mask[u][v] (the general token-level M of
+        Eq. 4 inside the chunk); a further mask on top of the others.
 
     Steps (Section 3.2): select the context states of the node with Eq. 2-3;
     rotate the K of the node's own state and of every selected state and the
@@ -268,12 +271,17 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
     row_frame = rows // frame_tokens if within == "frame_causal" else np.zeros_like(rows)
     row_tile = rows // 128 if tile_mask is not None else np.zeros_like(rows)
     groups = []
-    for f in np.unique(row_frame):
-        for qt in np.unique(row_tile):
-            idx = np.nonzero((row_frame == f) & (row_tile == qt))[0]
-            if len(idx):
-                groups.append((f if within == "frame_causal" else None,
-                               qt if tile_mask is not None else None, idx))
+    if own_mask is not None:       # every row its own mask
+        for r in range(len(rows)):
+            groups.append((row_frame[r] if within == "frame_causal" else None,
+                           row_tile[r] if tile_mask is not None else None, np.array([r])))
+    else:
+        for f in np.unique(row_frame):
+            for qt in np.unique(row_tile):
+                idx = np.nonzero((row_frame == f) & (row_tile == qt))[0]
+                if len(idx):
+                    groups.append((f if within == "frame_causal" else None,
+                                   qt if tile_mask is not None else None, idx))
     if norm is not None:
         gk, gq, eps = norm
         states = {s: (rms_norm(states[s][0], gk, eps), states[s][1])
@@ -298,6 +306,9 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
                 for si in range(len(key_states)):
                     kept = np.asarray(tile_mask[qt][si * nt + key_tile], dtype=bool)
                     m[si * g.T:(si + 1) * g.T] = np.where(kept, m[si * g.T:(si + 1) * g.T], -np.inf)
+            if own_mask is not None:
+                u = rows[idx[0]]
+                m[:g.T] = np.where(np.asarray(own_mask[u], dtype=bool), m[:g.T], -np.inf)
             o, l = attend_rows(q[idx], k, v, scale, m)
             out[hi, idx] = o
             lse[hi, idx] = l

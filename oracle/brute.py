@@ -72,7 +72,7 @@ def _rope(x: np.ndarray, chunk: int, F: int, Hp: int, Wp: int, pairs, theta: flo
 def brute_forward(policy: str, W: int, F: int, Hp: int, Wp: int, pairs, theta: float,
                   node: tuple[int, int, int], grid: dict, q_raw: np.ndarray,
                   heads, scale: float, hidden=frozenset(), frame_causal: bool = False,
-                  tile_mask=None):
+                  tile_mask=None, own_mask=None):
     """All query rows of `heads` for node (seq, b, j) against the whole grid.
 
     grid: {(seq, chunk, level): (K_raw, V_raw)} [T][H][d]; it may hold states
@@ -83,6 +83,8 @@ def brute_forward(policy: str, W: int, F: int, Hp: int, Wp: int, pairs, theta: f
     tile_mask: None, or booleans [query tile][key tile]: query u sees key
     token v of state (c, l) only if entry [u // 128][r * nt + v // 128] is
     set, r = b - c (the offset of Eq. 2; 0 for the own chunk), nt = ceil(T/128).
+    own_mask: None, or booleans [T][T]: query u sees key token v of its own
+    chunk only if own_mask[u][v].
     Returns (out [len(heads)][T][d], lse [len(heads)][T]).
     """
     seq, b, j = node
@@ -113,6 +115,10 @@ def brute_forward(policy: str, W: int, F: int, Hp: int, Wp: int, pairs, theta: f
             if frame_causal:
                 for v in range(T):
                     if v // (Hp * Wp) > u // (Hp * Wp):
+                        Mu[own_start + v] = -np.inf
+            if own_mask is not None:
+                for v in range(T):
+                    if not own_mask[u][v]:
                         Mu[own_start + v] = -np.inf
             if tile_mask is not None:
                 for ki, (s, c, l) in enumerate(keys):

@@ -266,3 +266,67 @@ def test_tile_mask_special_cases(oracle_mod):
                                        tile_mask=none_for_tile1)
     assert np.all(c[:, 128:256] == 0.0) and np.all(lc[:, 128:256] == -np.inf)
     np.testing.assert_array_equal(c[:, :128], dense[:, :128])
+
+
+def _own_mask(T, seed, density=0.5):
+    rng = np.random.default_rng(seed)
+    m = rng.random((T, T)) < density
+    np.fill_diagonal(m, True)
+    m[5, :] = False                            # row 5 sees no key of its own chunk
+    return m
+
+
+@pytest.mark.parametrize("within", ["bidirectional", "frame_causal"])
+def test_own_token_mask_against_dense_brute_force(oracle_mod, within):
+    from oracle import brute
+    w, inp, g, states, masks = _sparse_case(oracle_mod, within)
+    rng = np.random.default_rng(6)
+    grid = dict(states)
+    for s in [(0, 2, 0), (0, 4, 0)]:
+        grid[s] = (rng.standard_normal((w.T, w.H, w.d)), rng.standard_normal((w.T, w.H, w.d)))
+    scale = 1.0 / math.sqrt(w.d)
+    rows = [0, 1, 5, 64, 127, 128, 200, 255, 256, 300, w.T - 1]
+    for i, node in enumerate(w.nodes):
+        own = _own_mask(w.T, 10 + i)
+        q = _f64(inp.q[i])
+        for tm in (None, masks[i]):
+            out, lse, _ = oracle_mod.node_forward(g, oracle_mod.POLICY_IDS[w.policy], w.W, node, states,
+                                                  q, range(w.H), rows, scale, within=within,
+                                                  tile_mask=tm, own_mask=own)
+            bo, bl = brute.brute_forward(w.policy, w.W, w.F, w.Hp, w.Wp, w.pairs, w.theta, node, grid,
+                                         q, range(w.H), scale, frame_causal=within == "frame_causal",
+                                         tile_mask=tm, own_mask=own)
+            np.testing.assert_allclose(out, bo[:, rows], rtol=0, atol=1e-12)
+            np.testing.assert_allclose(lse, bl[:, rows], rtol=0, atol=1e-12)
+
+
+def test_own_token_mask_special_cases(oracle_mod):
+    """An all-true own mask is the unmasked node; the lower-triangular-by-frame
+    own mask is the frame-causal mode; a row whose own mask is all false sees
+    only the history."""
+    w, inp, g, states, _ = _sparse_case(oracle_mod, "bidirectional")
+    pol = oracle_mod.POLICY_IDS[w.policy]
+    node = w.nodes[0]
+    q = _f64(inp.q[0])
+    rows = [0, 5, 130, w.T - 1]
+    base, bl, sel = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), rows, 0.125)
+    a, la, _ = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), rows, 0.125,
+                                       own_mask=np.ones((w.T, w.T), bool))
+    np.testing.assert_array_equal(a, base)
+    # frame-causal as a token mask (frames of 160 tokens in the two-frame variant)
+    w2, inp2, g2, states2, _ = _sparse_case(oracle_mod, "frame_causal")
+    q2 = _f64(inp2.q[0])
+    ft = w2.Hp * w2.Wp
+    fc = (np.arange(w2.T)[None, :] // ft) <= (np.arange(w2.T)[:, None] // ft)
+    x, lx, _ = oracle_mod.node_forward(g2, pol, w2.W, w2.nodes[0], states2, q2, range(w2.H), rows, 0.125,
+                                       within="frame_causal")
+    y, ly, _ = oracle_mod.node_forward(g2, pol, w2.W, w2.nodes[0], states2, q2, range(w2.H), rows, 0.125,
+                                       own_mask=fc)
+    np.testing.assert_array_equal(x, y)
+    # no own key: the row attends the history alone, i.e. the node with its own
+    # state hidden from that row
+    none = np.ones((w.T, w.T), bool)
+    none[130, :] = False
+    z, lz, _ = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), [130], 0.125,
+                                       own_mask=none)
+    assert not np.allclose(z, base[:, 2:3])
