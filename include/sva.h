@@ -262,6 +262,35 @@ sva_status sva_attend_nodes_sparse(sva_cache* c, const sva_node* nodes, int32_t 
                                    const uint32_t* tile_mask, int32_t words_per_row,
                                    sva_stream s);
 
+/* The masks of sva_attend_nodes_masked, both optional (NULL: no such mask). */
+typedef struct {
+  /* Block-sparse access, as the tile_mask / words_per_row of
+   * sva_attend_nodes_sparse. */
+  const uint32_t* tile_mask;
+  int32_t tile_words;
+  /* Token-level visibility inside each node's own chunk: device array of
+   * 32-bit words [n_nodes][T][own_words]; bit v (word v / 32, bit v % 32) of
+   * row (node i, query token u) set means query u of node i may attend key
+   * token v of its own chunk.  own_words >= ceil(T / 32); 4-byte aligned. */
+  const uint32_t* own_mask;
+  int32_t own_words;
+} sva_attn_mask;
+
+/* sva_attend_nodes with the general token-level mask M of Eq. 4 (Section
+ * 3.2) inside the own chunk and/or query-dependent block-sparse access to
+ * the history: M(u, v) = -inf where the own-chunk bit of (u, v) or the tile
+ * bit of (u's query tile, v's key tile) is clear, on top of every other mask
+ * (hidden context slots, the within-chunk mode, padding).  The frame-causal
+ * mode is the own mask with bit v set iff v's latent frame is not after u's.
+ * Queries that see no key get O = 0 and LSE = -inf.  Both masks are read by
+ * the kernel on `s` and must stay valid until it completes.  Errors: as
+ * sva_attend_nodes_sparse, plus INVALID_ARGUMENT for a misaligned own mask
+ * or a short own row; a NULL mask pointer or two NULL masks is plain
+ * sva_attend_nodes. */
+sva_status sva_attend_nodes_masked(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
+                                   const void* q, void* out, float* lse, float scale,
+                                   const sva_attn_mask* mask, sva_stream s);
+
 /* Bytes of the optional split workspace of a cache (0 if c is NULL).  With
  * a workspace attached, sva_attend_nodes may divide each (node, head,
  * query-tile pair) work unit into up to 4 contiguous key ranges computed by

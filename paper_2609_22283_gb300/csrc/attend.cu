@@ -228,10 +228,12 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
   if constexpr (sparse) if (warp == 2) {
     // Gather the caller's mask rows of the two query tiles into the kernel's
     // key tile order (slot list without hidden context slots), then take
-    // this split's share of the union's set bits.
+    // this split's share of the union's set bits.  Without a tile mask every
+    // key tile is kept.
     const int words = (n_all + 31) >> 5;  // <= kMaskWords, checked on the host
-    const uint32_t* row0 = p.tile_mask + ((size_t)nd.q_index * p.n_qt + qt0) * p.mask_words;
-    const uint32_t* row1 = row0 + p.mask_words;
+    const uint32_t* row0 =
+        p.tile_mask ? p.tile_mask + ((size_t)nd.q_index * p.n_qt + qt0) * p.mask_words : nullptr;
+    const uint32_t* row1 = row0 ? row0 + p.mask_words : nullptr;
     int total = 0;
     for (int w = 0; w < words; ++w) {
       const int i = (w << 5) + lane;
@@ -239,8 +241,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       if (i < n_all) {
         const int s = i / p.nt_slot;
         const int k = nd.src[s] * p.nt_slot + (i - s * p.nt_slot);
-        b0 = (row0[k >> 5] >> (k & 31)) & 1u;
-        if (has_q1) b1 = (row1[k >> 5] >> (k & 31)) & 1u;
+        b0 = row0 ? ((row0[k >> 5] >> (k & 31)) & 1u) != 0u : true;
+        if (has_q1) b1 = row1 ? ((row1[k >> 5] >> (k & 31)) & 1u) != 0u : true;
       }
       const uint32_t m0 = __ballot_sync(0xffffffffu, b0);
       const uint32_t m1 = __ballot_sync(0xffffffffu, b1);
@@ -509,6 +511,19 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
 #pragma unroll
       for (int b = 0; b < 2; ++b) {
         if (b == 1 && !has_q1) break;
+        // own-chunk token mask (masked instance): this thread's 64 bits of its
+        // row, fetched before the wait so that the load hides behind it
+        const bool own_tile = sparse && p.own_mask != nullptr && kt < p.nt_slot;
+        uint32_t ow[2] = {~0u, ~0u};
+        if (own_tile) {
+          const int u = (qt0 + b) * kTile + row;
+          if (u < p.T) {  // rows past T are never stored
+            const uint32_t* mrow = p.own_mask + ((size_t)nd.q_index * p.T + u) * p.own_words;
+            const int wi = kt * 4 + half * 2;  // word holding key 128 kt + 64 half
+            ow[0] = wi < p.own_words ? __ldg(mrow + wi) : 0u;
+            ow[1] = wi + 1 < p.own_words ? __ldg(mrow + wi + 1) : 0u;
+          }
+        }
         ok = mbar_wait(&bars.s_full[b], (uint32_t)i & 1u, &abort_flag, tmo);
         ok = __all_sync(0xffffffffu, ok);
         if (!ok) break;
@@ -543,13 +558,13 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         // Tiles that can hold masked keys (a slot's ragged last tile, the own
         // chunk under frame causality) take the masked path; the test is the
         // same for every thread, so it needs no vote.
-        if (valid_tile < kTile || own_fc) {
+        if (valid_tile < kTile || own_fc || own_tile) {
           float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
           for (int c = 0; c < 2; ++c)
 #pragma unroll
             for (int e = 0; e < 32; ++e)
-              if (c * 32 + e >= vrel) s[c][e] = __float_as_uint(-INFINITY);
+              if (c * 32 + e >= vrel || !((ow[c] >> e) & 1u)) s[c][e] = __float_as_uint(-INFINITY);
 #pragma unroll
           for (int c = 0; c < 2; ++c)
 #pragma unroll
@@ -566,7 +581,10 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         const float m_new = fmaxf(m[b], m_tile);
         const bool need = m_new > m[b] + kRescaleThreshold;
         if (__any_sync(0xffffffffu, need)) {
-          const float alpha = ex2(m[b] - m_new);  // 0 on the first tile (m = -inf)
+          // 0 when the row's first visible keys arrive (m = -inf); 1 for a row
+          // of the warp whose max did not move (also when it is still -inf:
+          // -inf - -inf would be NaN)
+          const float alpha = m_new > m[b] ? ex2(m[b] - m_new) : 1.0f;
           if (sparse ? o_has[b] : i > 0) {
             // O_b holds the sum over earlier tiles: the commit that completed
             // S_b of this tile came after PV_b of the previous one.
@@ -804,7 +822,7 @@ cudaError_t launch_d(const AttnParams& p, int grid, cudaStream_t s) {
     }
     configured[dev] = true;
   }
-  if (p.tile_mask != nullptr)
+  if (p.masked)
     attend_kernel<D, true><<<grid, kThreads, C::kSmemBytes, s>>>(p);
   else
     attend_kernel<D, false><<<grid, kThreads, C::kSmemBytes, s>>>(p);

@@ -57,6 +57,9 @@ struct alignas(128) AttnParams {
   uint64_t timeout_ns;
   const uint32_t* tile_mask;  // block-sparse visibility [n_nodes][n_qt][mask_words], or null
   int32_t mask_words;
+  const uint32_t* own_mask;   // token visibility in the own chunk [n_nodes][T][own_words], or null
+  int32_t own_words;
+  int32_t masked;             // tile_mask or own_mask given: the masked kernel instance
   AttnNode nodes[SVA_MAX_NODES];
 };
 

@@ -582,10 +582,10 @@ sva_status sva_rope_kv_write_qknorm(sva_cache* c, const sva_node* nodes, int32_t
 namespace {
 
 // sva_attend_nodes and sva_attend_nodes_sparse: the checks and the launch;
-// tile_mask NULL is the dense mask.
+// tile_mask and own_mask NULL is the dense mask.
 sva_status attend(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* q, void* out,
                   float* lse, float scale, const uint32_t* tile_mask, int32_t mask_words,
-                  sva_stream s) {
+                  const uint32_t* own_mask, int32_t own_words, sva_stream s) {
   if (c == nullptr || nodes == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "NULL argument");
   if (n_nodes < 1) return fail(SVA_ERR_INVALID_ARGUMENT, "n_nodes %d < 1", n_nodes);
   if (n_nodes > SVA_MAX_NODES)
@@ -658,6 +658,21 @@ sva_status attend(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const vo
     p.tile_mask = tile_mask;
     p.mask_words = mask_words;
   }
+  if (own_mask != nullptr) {
+    if ((reinterpret_cast<uintptr_t>(own_mask) & 3u) != 0)
+      return fail(SVA_ERR_INVALID_ARGUMENT, "own_mask must be 4-byte aligned");
+    if (own_words < (c->L.T + 31) / 32)
+      return fail(SVA_ERR_INVALID_ARGUMENT, "own_words %d < %d needed for %d tokens", own_words,
+                  (c->L.T + 31) / 32, c->L.T);
+    p.own_mask = own_mask;
+    p.own_words = own_words;
+  }
+  p.masked = (tile_mask != nullptr || own_mask != nullptr) ? 1 : 0;
+  if (p.masked)  // the masked kernel keeps a bitmap of the node's key tiles
+    for (int i = 0; i < n_nodes; ++i)
+      if ((long long)p.nodes[i].n_kv * p.nt_slot > 32LL * sva::kMaskWords)
+        return fail(SVA_ERR_CAPACITY, "node %d: %lld key tiles exceed the %d a masked launch covers",
+                    i, (long long)p.nodes[i].n_kv * p.nt_slot, 32 * sva::kMaskWords);
   if (c->q_cached != q || c->q_cached_n != n_nodes) {
     st = encode_4d_q(&c->tmap_q, q, g, c->L.T, n_nodes);
     if (st != SVA_OK) {
@@ -707,7 +722,7 @@ extern "C" {
 
 sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* q,
                             void* out, float* lse, float scale, sva_stream s) {
-  return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, s);
+  return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, s);
 }
 
 sva_status sva_qkv_project(sva_cache* c, const void* x, int32_t rows, int32_t in_features,
@@ -780,7 +795,15 @@ sva_status sva_attend_nodes_sparse(sva_cache* c, const sva_node* nodes, int32_t 
                                    const uint32_t* tile_mask, int32_t words_per_row,
                                    sva_stream s) {
   if (tile_mask == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "tile_mask is NULL");
-  return attend(c, nodes, n_nodes, q, out, lse, scale, tile_mask, words_per_row, s);
+  return attend(c, nodes, n_nodes, q, out, lse, scale, tile_mask, words_per_row, nullptr, 0, s);
+}
+
+sva_status sva_attend_nodes_masked(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
+                                   const void* q, void* out, float* lse, float scale,
+                                   const sva_attn_mask* mask, sva_stream s) {
+  if (mask == nullptr) return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, s);
+  return attend(c, nodes, n_nodes, q, out, lse, scale, mask->tile_mask, mask->tile_words,
+                mask->own_mask, mask->own_words, s);
 }
 
 // Attention with the split scratch taken from the library's own device

@@ -241,20 +241,37 @@ def tile_mask(w: Workload, density: float | None = None, seed: int | None = None
     return pack_bits(keep, w.mask_words)
 
 
+def own_mask(w: Workload, density: float, seed: int | None = None) -> torch.Tensor:
+    """Seeded token-level visibility inside each node's own chunk, int32
+    [n_nodes][T][ceil(T/32)] words: bit v of row (node, u) is kept when a
+    U(0, 1) draw (one per bit, row-major, on a generator seeded with `seed`,
+    default the workload's seed + 3000) is below `density`; the diagonal
+    (u sees itself) is always kept."""
+    g = torch.Generator(device="cpu")
+    g.manual_seed(w.seed + 3000 if seed is None else seed)
+    keep = torch.rand((w.n_nodes, w.T, w.T), generator=g, dtype=torch.float32) < density
+    idx = torch.arange(w.T)
+    keep[:, idx, idx] = True
+    return pack_bits(keep, -(-w.T // 32))
+
+
 def pack_bits(keep: torch.Tensor, words: int) -> torch.Tensor:
     """bool [..., nbits] -> int32 [..., words], bit k in word k // 32 at position k % 32."""
-    nbits = keep.shape[-1]
-    pad = torch.zeros(keep.shape[:-1] + (words * 32 - nbits,), dtype=torch.bool)
-    b = torch.cat([keep, pad], dim=-1).reshape(keep.shape[:-1] + (words, 32)).to(torch.int64)
-    v = (b << torch.arange(32, dtype=torch.int64)).sum(-1)
-    return torch.where(v >= 2 ** 31, v - 2 ** 32, v).to(torch.int32)
+    import numpy as np
+    k = np.ascontiguousarray(keep.numpy() if isinstance(keep, torch.Tensor) else keep, dtype=bool)
+    pad = words * 32 - k.shape[-1]
+    if pad:
+        k = np.concatenate([k, np.zeros(k.shape[:-1] + (pad,), dtype=bool)], axis=-1)
+    b = np.packbits(k, axis=-1, bitorder="little")            # bytes, little-endian bit order
+    return torch.from_numpy(np.ascontiguousarray(b).view("<i4").copy())
 
 
 def unpack_bits(words: torch.Tensor, nbits: int) -> torch.Tensor:
     """int32 [..., words] -> bool [..., nbits] (inverse of pack_bits)."""
-    v = words.to(torch.int64) & 0xFFFFFFFF
-    b = (v.unsqueeze(-1) >> torch.arange(32, dtype=torch.int64)) & 1
-    return b.reshape(words.shape[:-1] + (-1,))[..., :nbits].to(torch.bool)
+    import numpy as np
+    w = np.ascontiguousarray(words.numpy()).astype("<i4", copy=False)
+    b = np.unpackbits(w.view(np.uint8), axis=-1, bitorder="little")
+    return torch.from_numpy(b[..., :nbits].astype(bool))
 
 
 def projection_inputs(w: Workload, in_features: int, seed: int | None = None):

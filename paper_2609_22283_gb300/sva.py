@@ -38,7 +38,8 @@ MAX_NODES = 64
 EXPORTED = ("sva_cache_bytes", "sva_cache_create", "sva_cache_bind", "sva_cache_lookup",
             "sva_cache_release", "sva_select_context", "sva_pipeline_round", "sva_check_pipeline",
             "sva_rope_kv_write", "sva_rope_kv_write_qknorm", "sva_attend_nodes",
-            "sva_attend_nodes_sparse", "sva_qkv_project", "sva_attend_workspace_bytes",
+            "sva_attend_nodes_sparse", "sva_attend_nodes_masked", "sva_qkv_project",
+            "sva_attend_workspace_bytes",
             "sva_cache_set_workspace", "sva_attend_nodes_noalloc", "sva_poll_device_status",
             "sva_debug_inject", "sva_destroy", "sva_last_error")
 
@@ -61,6 +62,11 @@ class sva_node(ctypes.Structure):
                 ("own_slot", ctypes.c_int32), ("within", ctypes.c_int32),
                 ("n_ctx", ctypes.c_int32),
                 ("ctx_slot", ctypes.c_int32 * MAX_CTX), ("ctx_visible", ctypes.c_uint8 * MAX_CTX)]
+
+
+class sva_attn_mask(ctypes.Structure):
+    _fields_ = [("tile_mask", ctypes.c_void_p), ("tile_words", ctypes.c_int32),
+                ("own_mask", ctypes.c_void_p), ("own_words", ctypes.c_int32)]
 
 
 _lib = None
@@ -92,6 +98,7 @@ def load(path: str = LIB_PATH):
         "sva_attend_nodes": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
         "sva_attend_nodes_sparse": ([p, pn, i32, p, p, p, ctypes.c_float, p, i32, p], i32),
         "sva_qkv_project": ([p, p, i32, i32, p, p, p, p, p, p], i32),
+        "sva_attend_nodes_masked": ([p, pn, i32, p, p, p, ctypes.c_float, p, p], i32),
         "sva_attend_workspace_bytes": ([p], ctypes.c_size_t),
         "sva_attend_nodes_noalloc": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
         "sva_cache_set_workspace": ([p, p, ctypes.c_size_t], i32),
@@ -310,6 +317,35 @@ class Cache:
                                           ctypes.c_void_p(lse.data_ptr() if lse is not None else 0),
                                           float(scale), ctypes.c_void_p(tile_mask.data_ptr()),
                                           int(tile_mask.shape[2]),
+                                          ctypes.c_void_p(_stream_handle(stream)))
+        _check(st)
+
+    def attend_nodes_masked(self, nodes, q, out, lse=None, scale=None, tile_mask=None,
+                            own_mask=None, stream=None, check=True):
+        """sva_attend_nodes_masked: tile_mask as in attend_nodes_sparse, own_mask a
+        contiguous int32 CUDA tensor [n_nodes][T][words] of own-chunk token bits;
+        either may be None."""
+        n = len(nodes) if not isinstance(nodes, ctypes.Array) else None
+        arr = nodes if isinstance(nodes, ctypes.Array) else make_nodes(nodes)
+        count = n if n is not None else len(arr)
+        g = self.g
+        if check:
+            _tok_major(q, "q", count, self.T, g.num_heads, g.head_dim)
+            _tok_major(out, "out", count, self.T, g.num_heads, g.head_dim)
+        for t, nm, rows in ((tile_mask, "tile_mask", -(-self.T // 128)), (own_mask, "own_mask", self.T)):
+            if t is not None and (t.dtype != torch.int32 or not t.is_cuda or not t.is_contiguous()
+                                  or t.dim() != 3 or tuple(t.shape[:2]) != (count, rows)):
+                raise ValueError(f"{nm} must be a contiguous int32 CUDA tensor [{count}][{rows}][words]")
+        m = sva_attn_mask(ctypes.c_void_p(tile_mask.data_ptr() if tile_mask is not None else 0),
+                          int(tile_mask.shape[2]) if tile_mask is not None else 0,
+                          ctypes.c_void_p(own_mask.data_ptr() if own_mask is not None else 0),
+                          int(own_mask.shape[2]) if own_mask is not None else 0)
+        if scale is None:
+            scale = 1.0 / math.sqrt(g.head_dim)
+        st = _lib.sva_attend_nodes_masked(self.handle, arr, count, ctypes.c_void_p(q.data_ptr()),
+                                          ctypes.c_void_p(out.data_ptr()),
+                                          ctypes.c_void_p(lse.data_ptr() if lse is not None else 0),
+                                          float(scale), ctypes.byref(m),
                                           ctypes.c_void_p(_stream_handle(stream)))
         _check(st)
 

@@ -33,12 +33,14 @@ def oracle_masks(w: I.Workload, mask=None) -> np.ndarray:
     return I.unpack_bits(m, (1 + w.W) * w.tiles).numpy()
 
 
-def oracle_node(w, inp, states, node_index, heads, rows, hidden=frozenset(), tile_mask=None):
+def oracle_node(w, inp, states, node_index, heads, rows, hidden=frozenset(), tile_mask=None,
+                own_mask=None):
     g = oracle_geometry(w)
     q = inp.q[node_index].to(torch.float64).numpy()
     out, lse, _ = oracle.node_forward(g, oracle.POLICY_IDS[w.policy], w.W, w.nodes[node_index],
                                       states, q, list(heads), list(rows), 1.0 / math.sqrt(w.d),
                                       hidden=hidden, within=w.within, tile_mask=tile_mask,
+                                      own_mask=own_mask,
                                       norm=((inp.gamma_k.double().numpy(), inp.gamma_q.double().numpy(),
                                              inp.norm_eps) if w.qknorm else None))
     return out, lse

@@ -32,12 +32,26 @@ def _all_rows(oracle_mod, w):
     step.close()
 
 
+# T = 1000 in 10 frames of 100 tokens, one history chunk: 4 work units of 16
+# key tiles split 4 ways.  The range of own tiles 4-7 (keys 512..1023) holds
+# no visible key for rows 400..499 but some for rows 500..511, which share a
+# warp with rows 496..499: rows whose max is still -inf in a warp where others
+# rescale (the softmax must not form -inf - -inf).
+SPLITFC_WARP = I.Workload(name="splitfcwarp", seed=18, F=10, Hp=10, Wp=10, H=1, d=128, K=2, W=1,
+                          policy="prog", nodes=((0, 2, 1),), prefilled=((0, 1, 0),),
+                          within="frame_causal", description="masked and visible rows in one warp")
+
+
 def test_tiny_frame_causal_all_rows(oracle_mod):
     _all_rows(oracle_mod, I.WORKLOADS["tinyfc"])
 
 
 def test_split_range_inside_own_chunk(oracle_mod):
     _all_rows(oracle_mod, SPLITFC)
+
+
+def test_fully_masked_and_visible_rows_in_one_warp(oracle_mod):
+    _all_rows(oracle_mod, SPLITFC_WARP)
 
 
 def test_prog4_frame_causal_sampled(oracle_mod):
