@@ -13,19 +13,24 @@
 // in shared memory serves both query tiles.
 //   warp 0     TMA producer: Q0/Q1 once, then K and V tiles of the slot list
 //              into rings of shared-memory stages (128B swizzle);
-//   warp 1     MMA issuer (the whole warp runs the loop, one elected lane
-//              issues) and TMEM owner;
+//   warps 1, 3 MMA issuers, warp 1 for query tile 0 and warp 3 for query
+//              tile 1 (each whole warp runs its loop, one elected lane
+//              issues); warp 1 also owns TMEM;
 //   warps 4-11 softmax, all eight warps on one query tile at a time (Q0 then
 //              Q1 of every key tile): two threads per query row, 64 keys
 //              each; S from TMEM, fp32 online softmax in the log2 domain with
 //              a lazy rescale of O, P written back over S as bf16; then the
 //              epilogue (O / l to bf16 global, optional LSE).
 // TMEM columns: S0 [0,128), S1 [128,256), O0 [256, 256+d), O1 [384, 384+d).
-// MMA order per key tile i: PV0_i, S0_{i+1}, PV1_i, S1_{i+1}, so the softmax
-// of either query tile has the other tile's PV and S (two 128x128x128 MMAs)
-// to hide behind.  A commit that completes S_b of tile i also implies PV_b of
-// tile i-1 is complete (MMAs execute in issue order), so the rescale of O_b
-// needs no extra barrier.
+// Each issuer's order per key tile i is PV_b,i then S_b,i+1, so the softmax of
+// either query tile has the other tile's PV and S (two 128x128x128 MMAs) to
+// hide behind.  A tcgen05.mma costs its issuing warp nearly as long as the
+// tensor pipe takes to run it (about 60 of 64 cycles while the softmax warps
+// share the SM), so one issuer for both tiles left the pipe idle whenever it
+// waited on a barrier; two issuers on different sub-partitions each have half
+// the MMAs to issue.  A commit that completes S_b of tile i also implies PV_b
+// of tile i-1 is complete (one issuer per tile, MMAs of a thread execute in
+// issue order), so the rescale of O_b needs no extra barrier.
 // A unit may be split into n_split contiguous key ranges (when there are too
 // few units to fill the GPU's waves): each split CTA writes its normalised
 // partial O with its row max and sum to the workspace and bumps the unit's
@@ -205,8 +210,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
   if (threadIdx.x == 0) {
     abort_flag = 0;
     mbar_init(&bars.q_full, 1);
-    mbar_init(&bars.o_final, 1);
-    mbar_init(&bars.drain, 1);
+    mbar_init(&bars.o_final, 2);  // one commit per MMA issuer
+    mbar_init(&bars.drain, 2);
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bars.s_full[b], 1);
       mbar_init(&bars.p_full[b], 256);
@@ -339,8 +344,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         v_issued = j + 1;
       }
     }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
+  } else if (warp == 1 || warp == 3) {
+    // ------------------------------------------------------------ MMA issuers
     // The whole warp runs the loop (waits are voted warp-wide so every lane
     // takes the same branch); one elected lane issues each MMA and commit.
     {
@@ -363,12 +368,12 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       auto vis = [&](int b, int kt) {
         return !sparse || ((tmask[b][kt >> 5] >> (kt & 31)) & 1u) != 0u;
       };
-      bool pv_started[2] = {false, false};
+      bool pv_started = false;  // this issuer's query tile has a PV in O
       // S_b = Q_b K_i^T into TMEM buffer b
       auto issue_s = [&](int b, int i, bool v) {
         if (v) {
           const uint64_t kb = dK + (uint64_t)(i % C::kKStages) * kTileStep;
-          const uint64_t qb = dQ[b];
+          const uint64_t qb = b == 0 ? dQ[0] : dQ[1];
           const uint32_t dcol = tbase + col_s(b);
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
@@ -383,12 +388,12 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         const uint64_t vb = dV + (uint64_t)(i % C::kVStages) * kTileStep;
         const uint32_t ocol = tbase + col_o(b);
         const uint32_t pcol = tbase + col_s(b);
-        const uint32_t acc0 = (sparse ? pv_started[b] : i > 0) ? 1u : 0u;
+        const uint32_t acc0 = (sparse ? pv_started : i > 0) ? 1u : 0u;
 #pragma unroll
         for (int kk = 0; kk < kTile / 16; ++kk)
           mma_ts_warp(ocol, pcol + kk * 8, vb + (uint64_t)((kk * 2048) >> 4), idesc_pv,
                  kk > 0 ? 1u : acc0);
-        if (sparse) pv_started[b] = true;
+        if (sparse) pv_started = true;
       };
       auto wait = [&](uint64_t* bar, uint32_t parity) {
         return __all_sync(0xffffffffu, mbar_wait(bar, parity, &abort_flag, tmo));
@@ -396,40 +401,33 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       auto wait_k = [&](int i) {
         return wait(&bars.k_full[i % C::kKStages], (uint32_t)(i / C::kKStages) & 1u);
       };
+      const int bq = warp == 1 ? 0 : 1;  // the query tile this warp issues for
       bool ok = wait(&bars.q_full, 0);
-      int kt = t_begin;  // key tile of the node at iteration i
-      if (n_tiles > 0) {  // a block-sparse range may be empty: then only o_final is committed
-        ok = ok && wait_k(0);
-        if (ok) {
-          tc_fence_after();
-          issue_s(0, 0, vis(0, kt));
-          if (has_q1) issue_s(1, 0, vis(1, kt));
+      if (bq == 0 || has_q1) {
+        int kt = t_begin;  // key tile of the node at iteration i
+        if (n_tiles > 0) {  // a block-sparse range may be empty: then only o_final is committed
+          ok = ok && wait_k(0);
+          if (ok) {
+            tc_fence_after();
+            issue_s(bq, 0, vis(bq, kt));
+          }
         }
-      }
-      for (int i = 0; ok && i < n_tiles; ++i) {
-        const uint32_t par = (uint32_t)i & 1u;
-        const bool more = i + 1 < n_tiles;
-        const int kt_next = !more ? kt : (sparse ? next_tile(tmask, kt + 1, n_all) : kt + 1);
-        // V_i and K_{i+1} land long before the softmax hands over P_0, so
-        // their waits go first, off the path from P_0 to the next MMA.
-        if (!wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u) ||
-            (more && !wait_k(i + 1)) || !wait(&bars.p_full[0], par)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        if (vis(0, kt)) issue_pv(0, i);
-        if (more) issue_s(0, i + 1, vis(0, kt_next));
-        if (has_q1) {
-          if (!wait(&bars.p_full[1], par)) {
+        for (int i = 0; ok && i < n_tiles; ++i) {
+          const uint32_t par = (uint32_t)i & 1u;
+          const bool more = i + 1 < n_tiles;
+          const int kt_next = !more ? kt : (sparse ? next_tile(tmask, kt + 1, n_all) : kt + 1);
+          // V_i and K_{i+1} normally land before the softmax hands over P_b,
+          // so their waits go first, off the path from P_b to the next MMA.
+          if (!wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u) ||
+              (more && !wait_k(i + 1)) || !wait(&bars.p_full[bq], par)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          if (vis(1, kt)) issue_pv(1, i);
+          if (vis(bq, kt)) issue_pv(bq, i);
+          if (more) issue_s(bq, i + 1, vis(bq, kt_next));
+          kt = kt_next;
         }
-        if (more && has_q1) issue_s(1, i + 1, vis(1, kt_next));
-        kt = kt_next;
       }
       if (ok) {
         mma_commit_warp(&bars.o_final);
@@ -456,7 +454,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
           if (p.fault_mode == 1 && i == 1) continue;  // the copy the test hook withheld
           mbar_wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u, &zero, tmo);
         }
-      } else if (warp == 1) {
+      } else if (warp == 1 || warp == 3) {
         mma_commit_warp(&bars.drain);  // the same elected lane that issued the MMAs
         mbar_wait(&bars.drain, 0, &zero, tmo);
       }
@@ -495,12 +493,13 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
 #pragma unroll
     for (int b = 0; b < 2; ++b)
       frame_end[b] = ((qt0 + b) * kTile + row) / p.frame_tokens * p.frame_tokens + p.frame_tokens;
-    // The commit that completes the last S of key tile i (S_1, or S_0
-    // without a second query tile) follows every MMA that reads K stage i
-    // and every PV of tile i-1, so one softmax thread hands K stage i and V
-    // stage i-1 back to the producer as soon as it sees that S.  The MMA
-    // warp then commits only to the two S barriers per tile (a commit costs
-    // it about as long as an MMA issue).
+    // The softmax sees S_0 and then S_1 of key tile i complete.  S_b,i
+    // follows PV_b,i-1 in its issuer's order, so once both are seen every
+    // MMA that reads K stage i or V stage i-1 has completed, and one softmax
+    // thread hands both stages back to the producer when it sees the last S
+    // of the tile (S_1, or S_0 without a second query tile).  The MMA warps
+    // then commit only to their S barriers (a commit costs an issuer about
+    // as long as an MMA).
     const bool releaser = warp == 4 && lane == 0;
     bool ok = true;
     int kt = t_begin;  // key tile of the node
