@@ -13,6 +13,8 @@ rows) and is driven from here:
 * ``rope_head`` / ``bf16`` -- the 3D RoPE reading and the bf16 cache store.
 * ``attend_rows`` -- Eq. 4 masked softmax attention.
 * ``qkv_project`` -- the input projection producing q, k, v token-major.
+* ``qkv_project_rope`` -- that projection with the RoPE of q and k applied to
+  its unrounded outputs (the fused projection + cache write).
 * ``node_forward`` -- one denoising node end to end: its context selection,
   the rotation of every key state it reads and of its queries, the bf16
   rounding of what the cache would hold, and the attention of the requested
@@ -193,6 +195,27 @@ def qkv_project(x: np.ndarray, weight: np.ndarray, bias=None, heads: int = 1):
     if bias is not None:
         y = y + np.asarray(bias, dtype=np.float64)[None, :]
     return tuple(y[:, t * n:(t + 1) * n].reshape(rows, heads, n // heads) for t in range(3))
+
+
+def qkv_project_rope(x: np.ndarray, weight: np.ndarray, bias, g: Geometry, chunks):
+    """The projection followed by the 3D RoPE of q and k, with no rounding in
+    between (the fused projection + RoPE + cache write), fp64.
+
+    x: [n * T][C], node i's token rows at [i*T, (i+1)*T); chunks[i] is node
+    i's chunk index (its tokens sit at frames F*chunks[i] + f).  Returns
+    (q', k', v), each [n][T][H][d], unrounded: q and k of every head rotated by
+    ``rope_head`` at the node's chunk, v as projected.
+    """
+    n = len(chunks)
+    q, k, v = qkv_project(x, weight, bias, heads=g.H)
+    shape = (n, g.T, g.H, g.d)
+    q, k, v = q.reshape(shape), k.reshape(shape), v.reshape(shape)
+    qr, kr = np.empty(shape), np.empty(shape)
+    for i, b in enumerate(chunks):
+        for h in range(g.H):
+            qr[i, :, h] = rope_head(q[i, :, h], b, g)
+            kr[i, :, h] = rope_head(k[i, :, h], b, g)
+    return qr, kr, v
 
 
 # ---------------------------------------------------------------- attention
