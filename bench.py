@@ -493,6 +493,12 @@ def run_ours(args, world, rank, local):
         # write, attention (kernel times summed; the projection is not in `value`)
         line["nodes_per_s_with_projection"] = (
             w.n_nodes * world / ((line["qkv_project"]["ms"] + t_step_ms) * 1e-3))
+        # the same layer with the RoPE + cache write fused into the projection
+        # (sva_qkv_project_rope, then the attention)
+        line["qkv_project_rope"] = time_projection(step, w, dev, flush, stream, peak, world,
+                                                   fused=True)
+        line["nodes_per_s_fused_layer"] = (
+            w.n_nodes * world / ((line["qkv_project_rope"]["ms"] + t_attn_ms) * 1e-3))
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         tf, rows, secs, cores = oracle_sample(w, inp, args.cpu_seconds)
         line["cpu_baseline"] = {
@@ -505,26 +511,36 @@ def run_ours(args, world, rank, local):
     return 0
 
 
-def time_projection(step, w, dev, flush, stream, peak, world):
+def time_projection(step, w, dev, flush, stream, peak, world, fused=False):
     """The input projection in front of the step (sva_qkv_project: [q | k | v] =
     x W^T + b for the step's n*T token rows, hidden size H*d), timed like the
     step: CUDA events per launch, L2 flushed between launches.  Reported
-    beside the step, not inside it."""
+    beside the step, not inside it.  With `fused`, sva_qkv_project_rope: the
+    same projection with the RoPE + cache write in its epilogue (it writes the
+    nodes' own slots; run after every timed step and check)."""
     import torch
     from paper_2609_22283_gb300 import inputs as I
     C = w.H * w.d
     x, wt, b = I.projection_inputs(w, C)
     x, wt, b = x.to(dev), wt.to(dev), b.to(dev)
     outs = [torch.empty((w.n_nodes, w.T, w.H, w.d), dtype=torch.bfloat16, device=dev) for _ in range(3)]
+    nodes, _ = step.node_table()
+
+    def launch():
+        if fused:
+            step.cache.qkv_project_rope(nodes, x, wt, b, outs[0], check=False)
+        else:
+            step.cache.qkv_project(x, wt, b, *outs, check=False)
+
     for _ in range(3):
-        step.cache.qkv_project(x, wt, b, *outs, check=False)
+        launch()
     K = 20
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(K)]
     torch.cuda.synchronize()
     for e0, e1 in ev:
         flush()
         e0.record(stream)
-        step.cache.qkv_project(x, wt, b, *outs, check=False)
+        launch()
         e1.record(stream)
     torch.cuda.synchronize()
     if step.cache.poll() != 0:
@@ -532,7 +548,8 @@ def time_projection(step, w, dev, flush, stream, peak, world):
     ms = reduce_max(sum(a.elapsed_time(c) for a, c in ev) / K, world)
     flops = 2.0 * w.n_nodes * w.T * C * 3 * C
     tf = flops / (ms * 1e-3) / 1e12
-    return {"kernel": "qkv_project_kernel", "rows": w.n_nodes * w.T, "in_features": C,
+    return {"kernel": "qkv_project_kernel" + (" (fused RoPE + cache write)" if fused else ""),
+            "rows": w.n_nodes * w.T, "in_features": C,
             "out_features": 3 * C, "ms": ms, "achieved": tf, "unit": "TFLOP/s",
             "peak": peak, "frac": tf / peak, "launches": K}
 

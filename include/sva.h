@@ -126,7 +126,8 @@ typedef struct {
 
 /* Bytes of device memory the cache needs for `g`: the slot pool
  * [num_slots][2 (K, V)][H][Tpad][d] bf16 with Tpad = T rounded up to 128,
- * the RoPE cos/sin tables and a status word.  0 if `g` is invalid. */
+ * the RoPE cos/sin tables (the patch-row and patch-column ones also stored
+ * pair-major) and a status word.  0 if `g` is invalid. */
 size_t sva_cache_bytes(const sva_geometry* g);
 
 /* Creates a cache over the caller's device buffer `dev_buf` (at least
@@ -219,6 +220,25 @@ sva_status sva_rope_kv_write_qknorm(sva_cache* c, const sva_node* nodes, int32_t
 sva_status sva_qkv_project(sva_cache* c, const void* x, int32_t rows, int32_t in_features,
                            const void* weight, const float* bias, void* q, void* k, void* v,
                            sva_stream s);
+
+/* sva_qkv_project with the RoPE + cache write of sva_rope_kv_write fused into
+ * its epilogue (no normalisation), for the token rows of n_nodes nodes:
+ * rows = n_nodes * T, node i's tokens at rows [i*T, (i+1)*T) of x.
+ *   [q | k | v] = x W^T + b        (fp32 accumulators, bias added in fp32)
+ * then q and k of each token are rotated by the 3D RoPE at its absolute
+ * position (F*chunk + f, h, w) in fp32 and rounded to bf16 once; Q' goes to
+ * q_out and K' with the unrotated V into each node's own slot, which is
+ * marked resident.  The result equals sva_qkv_project followed by
+ * sva_rope_kv_write up to the intermediate bf16 rounding of q and k, which
+ * this call does not make.
+ *   nodes   as for sva_rope_kv_write (own_slot bound to (seq, chunk, level),
+ *           distinct own slots, n_nodes <= SVA_MAX_NODES)
+ *   x       [n_nodes*T][in_features] bf16; weight, bias as sva_qkv_project
+ *   q_out   [n_nodes][T][H][d] bf16
+ * Stream-ordered.  Errors: those of sva_qkv_project and sva_rope_kv_write. */
+sva_status sva_qkv_project_rope(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
+                                const void* x, int32_t in_features, const void* weight,
+                                const float* bias, void* q_out, sva_stream s);
 
 /* Policy-indexed chunk-causal attention (Eq. 4) for a batch of nodes:
  *   out[i][u][h] = sum_v softmax_v(scale * q[i][u][h] . k_v + M(u, v)) v_v

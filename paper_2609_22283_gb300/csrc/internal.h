@@ -97,6 +97,13 @@ struct ProjParams {
   int32_t rows, C, N;  // N = H * d outputs per tensor
   int32_t n_mtiles, n_ntiles, n_kblocks;
   uint64_t timeout_ns;
+  // Fused RoPE + cache scatter epilogue (sva_qkv_project_rope): q and k are
+  // rotated in fp32 before their one bf16 rounding, Q' goes to out[0], K' and
+  // V into the nodes' own slots (rope.cache, rope.nodes); out[1], out[2] and
+  // rope.k_new / v_new / q are unused; rope.tab_h and rope.tab_w point at the
+  // pair-major copies of those tables.  rows = rope.n_nodes * rope.T.
+  int32_t rope_on;
+  RopeParams rope;
 };
 
 cudaError_t launch_qkv_project(const ProjParams& p, int block_n, int grid, cudaStream_t s);

@@ -19,7 +19,10 @@
 //   warp 1     TMEM owner and MMA issuer (whole warp, one elected lane);
 //   warps 4-7  epilogue, one output row per thread.
 // A tile never straddles q, k and v (N is a multiple of BN), so its epilogue
-// writes into one tensor.  Rows past `rows` read zeros (TMA fill) and are
+// writes into one tensor.  With the fused RoPE epilogue (sva_qkv_project_rope)
+// each thread rotates the pairs of its row's q and k columns in fp32 at the
+// token's (t, h, w) position before the one bf16 rounding, writes Q' token-
+// major and scatters K' and V into the node's own cache slot.  Rows past `rows` read zeros (TMA fill) and are
 // not stored; K past C reads zeros on both operands.  All waits are bounded:
 // on expiry the CTA records SVA_ERR_DEVICE_TIMEOUT, drains its own copies and
 // MMAs, frees TMEM and exits.
@@ -92,6 +95,23 @@ __device__ __forceinline__ void mma_commit_mc_warp(uint64_t* bar, uint16_t mask)
       " @e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n"
       "}\n" ::"r"(smem_u32(bar)), "h"(mask)
       : "memory");
+}
+
+// (cos, sin) of pair `pi` of a head at position (t, hh, ww): pairs [0, P0)
+// rotate with the frame index, [P0, P0+P1) with the patch row, the rest with
+// the patch column (the same values and split as the RoPE + cache write).
+// Here the patch-row and patch-column tables are the pair-major copies
+// ([pair][position]), so the 32 tokens of a warp read neighbouring entries.
+__device__ __forceinline__ float2 rope_cs(const RopeParams& r, int pi, int t, int hh, int ww) {
+  if (pi < r.P0) return __ldg(r.tab_t + (size_t)t * r.P0 + pi);
+  if (pi < r.P0 + r.P1) return __ldg(r.tab_h + (size_t)(pi - r.P0) * r.Hp + hh);
+  return __ldg(r.tab_w + (size_t)(pi - r.P0 - r.P1) * r.Wp + ww);
+}
+
+__device__ __forceinline__ uint32_t rotate2_bf16(float x, float y, float2 cs) {
+  const float rx = __fmaf_rn(x, cs.x, -(y * cs.y));
+  const float ry = __fmaf_rn(x, cs.y, y * cs.x);
+  return pack2_bf16(rx, ry);
 }
 
 __device__ __forceinline__ void proj_timeout(const ProjParams& p, volatile int* abort_flag) {
@@ -238,13 +258,26 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
       const int c0 = col - tensor * p.N;  // column inside that tensor
       const long long grow = (long long)m * kBM + row;
       const bool in_range = grow < p.rows;
-      __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.out[tensor]) + grow * p.N + c0;
-#pragma unroll 1
-      for (int c = 0; c < BN / 32; ++c) {
-        uint32_t r[32];
+      __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.out[p.rope_on ? 0 : tensor]) + grow * p.N + c0;
+      // fused RoPE: this row's node, token and position, and where K' / V go
+      int tpos = 0, hh = 0, ww = 0;
+      __nv_bfloat16* cdst = nullptr;  // (slot, K or V, head 0, token u, dim 0) of the cache
+      if (p.rope_on && in_range) {
+        const RopeParams& rp = p.rope;
+        const int node = (int)(grow / rp.T);
+        const int u = (int)(grow - (long long)node * rp.T);
+        const int HpWp = rp.Hp * rp.Wp;
+        const int f = u / HpWp;
+        hh = (u - f * HpWp) / rp.Wp;
+        ww = u - f * HpWp - hh * rp.Wp;
+        tpos = rp.nodes[node].t_base + f;
+        cdst = static_cast<__nv_bfloat16*>(rp.cache) +
+               ((((size_t)rp.nodes[node].slot * 2 + (tensor == 2 ? 1 : 0)) * rp.H) * rp.Tpad + u) * rp.d;
+      }
+      // 32 accumulator columns of this row: TMEM -> registers, plus the bias
+      auto load_chunk = [&](int c, uint32_t (&r)[32], float (&bv)[32]) {
         tmem_ld32(tbase + lane_off + (uint32_t)(acc * BN + c * 32), r);
         tmem_wait_ld(r);
-        float bv[32];
         if (p.bias != nullptr) {
           const float4* b4 = reinterpret_cast<const float4*>(p.bias + col + c * 32);
 #pragma unroll
@@ -256,16 +289,62 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
 #pragma unroll
           for (int e = 0; e < 32; ++e) bv[e] = 0.0f;
         }
-        if (in_range) {
-          uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
+      };
+      if (p.rope_on) {
+        // Fused RoPE: the 32-column chunk ci of every head in the tile uses
+        // the same 16 (cos, sin) pairs, fetched once.
+        const RopeParams& rp = p.rope;
+        const int cpd = rp.d / 32;  // chunks per head
+#pragma unroll 1
+        for (int ci = 0; ci < cpd; ++ci) {
+          float2 cs[16];
+          if (tensor != 2) {
 #pragma unroll
-          for (int v = 0; v < 4; ++v) {
-            uint4 w;
-            w.x = pack2_bf16(__uint_as_float(r[8 * v + 0]) + bv[8 * v + 0], __uint_as_float(r[8 * v + 1]) + bv[8 * v + 1]);
-            w.y = pack2_bf16(__uint_as_float(r[8 * v + 2]) + bv[8 * v + 2], __uint_as_float(r[8 * v + 3]) + bv[8 * v + 3]);
-            w.z = pack2_bf16(__uint_as_float(r[8 * v + 4]) + bv[8 * v + 4], __uint_as_float(r[8 * v + 5]) + bv[8 * v + 5]);
-            w.w = pack2_bf16(__uint_as_float(r[8 * v + 6]) + bv[8 * v + 6], __uint_as_float(r[8 * v + 7]) + bv[8 * v + 7]);
-            d4[v] = w;
+            for (int e = 0; e < 16; ++e) cs[e] = rope_cs(rp, ci * 16 + e, tpos, hh, ww);
+          }
+#pragma unroll 1
+          for (int hb = 0; hb < BN / rp.d; ++hb) {
+            const int c = hb * cpd + ci;
+            uint32_t r[32];
+            float bv[32];
+            load_chunk(c, r, bv);  // warp-collective: every thread, in range or not
+            if (in_range) {
+              const int head = (c0 + c * 32) / rp.d;
+              uint32_t w[16];
+              if (tensor == 2) {
+#pragma unroll
+                for (int e = 0; e < 16; ++e)
+                  w[e] = pack2_bf16(__uint_as_float(r[2 * e]) + bv[2 * e], __uint_as_float(r[2 * e + 1]) + bv[2 * e + 1]);
+              } else {
+#pragma unroll
+                for (int e = 0; e < 16; ++e)
+                  w[e] = rotate2_bf16(__uint_as_float(r[2 * e]) + bv[2 * e],
+                                      __uint_as_float(r[2 * e + 1]) + bv[2 * e + 1], cs[e]);
+              }
+              uint4* d4 = reinterpret_cast<uint4*>(
+                  tensor == 0 ? dst + c * 32 : cdst + (size_t)head * rp.Tpad * rp.d + ci * 32);
+#pragma unroll
+              for (int v = 0; v < 4; ++v) d4[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
+            }
+          }
+        }
+      } else {
+#pragma unroll 1
+        for (int c = 0; c < BN / 32; ++c) {
+          uint32_t r[32];
+          float bv[32];
+          load_chunk(c, r, bv);  // warp-collective: every thread, in range or not
+          if (in_range) {
+            uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
+#pragma unroll
+            for (int v = 0; v < 4; ++v) {
+              uint4 w;
+              w.x = pack2_bf16(__uint_as_float(r[8 * v + 0]) + bv[8 * v + 0], __uint_as_float(r[8 * v + 1]) + bv[8 * v + 1]);
+              w.y = pack2_bf16(__uint_as_float(r[8 * v + 2]) + bv[8 * v + 2], __uint_as_float(r[8 * v + 3]) + bv[8 * v + 3]);
+              w.z = pack2_bf16(__uint_as_float(r[8 * v + 4]) + bv[8 * v + 4], __uint_as_float(r[8 * v + 5]) + bv[8 * v + 5]);
+              w.w = pack2_bf16(__uint_as_float(r[8 * v + 6]) + bv[8 * v + 6], __uint_as_float(r[8 * v + 7]) + bv[8 * v + 7]);
+              d4[v] = w;
+            }
           }
         }
       }

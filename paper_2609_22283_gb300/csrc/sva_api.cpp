@@ -6,6 +6,7 @@
 // descriptors, and the launches of the two kernels.  Device memory is always
 // the caller's.
 #include <algorithm>
+#include <climits>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -66,7 +67,7 @@ struct Layout {
   int T = 0;
   int Tpad = 0;
   size_t slot_bytes = 0;  // whole slot pool
-  size_t tab_t = 0, tab_h = 0, tab_w = 0, status = 0;  // byte offsets
+  size_t tab_t = 0, tab_h = 0, tab_w = 0, tab_ht = 0, tab_wt = 0, status = 0;  // byte offsets
   size_t total = 0;
 };
 
@@ -123,6 +124,12 @@ Layout layout_of(const sva_geometry& g) {
   L.tab_h = off;
   off = round_up(off + (size_t)g.grid_h * g.rope_pairs[1] * sizeof(float2), 256);
   L.tab_w = off;
+  off = round_up(off + (size_t)g.grid_w * g.rope_pairs[2] * sizeof(float2), 256);
+  // the patch-row and patch-column tables again, pair-major ([pair][position]),
+  // for readers whose neighbouring threads hold neighbouring tokens
+  L.tab_ht = off;
+  off = round_up(off + (size_t)g.grid_h * g.rope_pairs[1] * sizeof(float2), 256);
+  L.tab_wt = off;
   off = round_up(off + (size_t)g.grid_w * g.rope_pairs[2] * sizeof(float2), 256);
   L.status = off;
   L.total = off + 256;
@@ -349,10 +356,18 @@ sva_status sva_cache_create(const sva_geometry* g, void* dev_buf, size_t bytes, 
   auto tt = rope_table(g->max_frames, g->rope_pairs[0], g->rope_theta);
   auto th = rope_table(g->grid_h, g->rope_pairs[1], g->rope_theta);
   auto tw = rope_table(g->grid_w, g->rope_pairs[2], g->rope_theta);
+  auto transpose = [](const std::vector<float2>& t, int n_pos, int n_pair) {
+    std::vector<float2> r(t.size());
+    for (int i = 0; i < n_pos; ++i)
+      for (int j = 0; j < n_pair; ++j) r[(size_t)j * n_pos + i] = t[(size_t)i * n_pair + j];
+    return r;
+  };
+  auto tht = transpose(th, g->grid_h, g->rope_pairs[1]);
+  auto twt = transpose(tw, g->grid_w, g->rope_pairs[2]);
   struct Up {
     size_t off;
     const std::vector<float2>* v;
-  } ups[3] = {{L.tab_t, &tt}, {L.tab_h, &th}, {L.tab_w, &tw}};
+  } ups[5] = {{L.tab_t, &tt}, {L.tab_h, &th}, {L.tab_w, &tw}, {L.tab_ht, &tht}, {L.tab_wt, &twt}};
   for (auto& u : ups) {
     if (u.v->empty()) continue;
     e = cudaMemcpy(c->base + u.off, u.v->data(), u.v->size() * sizeof(float2),
@@ -725,19 +740,27 @@ sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes
   return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, s);
 }
 
-sva_status sva_qkv_project(sva_cache* c, const void* x, int32_t rows, int32_t in_features,
-                           const void* weight, const float* bias, void* q, void* k, void* v,
-                           sva_stream s) {
+}  // extern "C"
+
+namespace {
+
+// sva_qkv_project, and with `nodes` non-NULL sva_qkv_project_rope (k, v are
+// then unused: K' and V go to the nodes' own slots).
+sva_status project(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* x,
+                   int32_t rows, int32_t in_features, const void* weight, const float* bias,
+                   void* q, void* k, void* v, sva_stream s) {
   if (c == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "NULL cache");
   if (rows < 1 || in_features < 8 || in_features % 8 != 0)
     return fail(SVA_ERR_INVALID_ARGUMENT,
                 "rows %d must be >= 1 and in_features %d a positive multiple of 8", rows,
                 in_features);
-  if (x == nullptr || weight == nullptr || q == nullptr || k == nullptr || v == nullptr ||
-      !aligned16(x) || !aligned16(weight) || !aligned16(q) || !aligned16(k) || !aligned16(v) ||
+  const bool rope = nodes != nullptr;
+  if (x == nullptr || weight == nullptr || q == nullptr || !aligned16(x) || !aligned16(weight) ||
+      !aligned16(q) || (!rope && (k == nullptr || v == nullptr || !aligned16(k) || !aligned16(v))) ||
       (bias != nullptr && !aligned16(bias)))
     return fail(SVA_ERR_INVALID_ARGUMENT,
-                "x, weight, q, k, v (and bias if given) must be non-NULL and 16-byte aligned");
+                rope ? "x, weight, q_out (and bias if given) must be non-NULL and 16-byte aligned"
+                     : "x, weight, q, k, v (and bias if given) must be non-NULL and 16-byte aligned");
   sva_status st = check_device(c);
   if (st != SVA_OK) return st;
   const sva_geometry& g = c->g;
@@ -770,6 +793,40 @@ sva_status sva_qkv_project(sva_cache* c, const void* x, int32_t rows, int32_t in
     if (r != CUDA_SUCCESS)
       return fail(SVA_ERR_CUDA, "cuTensorMapEncodeTiled(weight) failed: %d", (int)r);
   }
+  if (rope) {
+    // the same node checks as sva_rope_kv_write
+    for (int i = 0; i < n_nodes; ++i) {
+      const sva_node& n = nodes[i];
+      st = check_own(c, n, i, false);
+      if (st != SVA_OK) return st;
+      for (int j = 0; j < i; ++j)
+        if (nodes[j].own_slot == n.own_slot)
+          return fail(SVA_ERR_INVALID_ARGUMENT, "nodes %d and %d write the same slot %d", j, i,
+                      n.own_slot);
+      const long long t0 = (long long)g.frames * n.chunk;
+      if (t0 < 0 || t0 + g.frames > g.max_frames)
+        return fail(SVA_ERR_CAPACITY,
+                    "node %d: chunk %d covers frames [%lld, %lld), outside the RoPE table [0, %d)",
+                    i, n.chunk, t0, t0 + g.frames, g.max_frames);
+      p.rope.nodes[i].slot = n.own_slot;
+      p.rope.nodes[i].t_base = (int32_t)t0;
+    }
+    p.rope_on = 1;
+    p.rope.cache = c->base;
+    p.rope.tab_t = reinterpret_cast<const float2*>(c->base + c->L.tab_t);
+    p.rope.tab_h = reinterpret_cast<const float2*>(c->base + c->L.tab_ht);  // pair-major
+    p.rope.tab_w = reinterpret_cast<const float2*>(c->base + c->L.tab_wt);  // pair-major
+    p.rope.T = c->L.T;
+    p.rope.H = g.num_heads;
+    p.rope.d = g.head_dim;
+    p.rope.Tpad = c->L.Tpad;
+    p.rope.Hp = g.grid_h;
+    p.rope.Wp = g.grid_w;
+    p.rope.P0 = g.rope_pairs[0];
+    p.rope.P1 = g.rope_pairs[1];
+    p.rope.P2 = g.rope_pairs[2];
+    p.rope.n_nodes = n_nodes;
+  }
   p.bias = bias;
   p.out[0] = q;
   p.out[1] = k;
@@ -787,7 +844,32 @@ sva_status sva_qkv_project(sva_cache* c, const void* x, int32_t rows, int32_t in
   const int grid = 2 * (int)std::min<long long>(pairs, c->num_sms / 2);
   cudaError_t e = sva::launch_qkv_project(p, bn, grid, reinterpret_cast<cudaStream_t>(s));
   if (e != cudaSuccess) return cuda_fail(e, "qkv_project launch");
+  if (rope)
+    for (int i = 0; i < n_nodes; ++i) c->slots[nodes[i].own_slot].resident = true;
   return ok();
+}
+
+}  // namespace
+
+extern "C" {
+
+sva_status sva_qkv_project(sva_cache* c, const void* x, int32_t rows, int32_t in_features,
+                           const void* weight, const float* bias, void* q, void* k, void* v,
+                           sva_stream s) {
+  return project(c, nullptr, 0, x, rows, in_features, weight, bias, q, k, v, s);
+}
+
+sva_status sva_qkv_project_rope(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
+                                const void* x, int32_t in_features, const void* weight,
+                                const float* bias, void* q_out, sva_stream s) {
+  if (c == nullptr || nodes == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "NULL argument");
+  if (n_nodes < 1) return fail(SVA_ERR_INVALID_ARGUMENT, "n_nodes %d < 1", n_nodes);
+  if (n_nodes > SVA_MAX_NODES)
+    return fail(SVA_ERR_CAPACITY, "n_nodes %d > SVA_MAX_NODES (%d)", n_nodes, SVA_MAX_NODES);
+  const long long rows = (long long)n_nodes * c->L.T;
+  if (rows > INT32_MAX) return fail(SVA_ERR_CAPACITY, "n_nodes * T = %lld rows", rows);
+  return project(c, nodes, n_nodes, x, (int32_t)rows, in_features, weight, bias, q_out, nullptr,
+                 nullptr, s);
 }
 
 sva_status sva_attend_nodes_sparse(sva_cache* c, const sva_node* nodes, int32_t n_nodes,

@@ -39,6 +39,7 @@ EXPORTED = ("sva_cache_bytes", "sva_cache_create", "sva_cache_bind", "sva_cache_
             "sva_cache_release", "sva_select_context", "sva_pipeline_round", "sva_check_pipeline",
             "sva_rope_kv_write", "sva_rope_kv_write_qknorm", "sva_attend_nodes",
             "sva_attend_nodes_sparse", "sva_attend_nodes_masked", "sva_qkv_project",
+            "sva_qkv_project_rope",
             "sva_attend_workspace_bytes",
             "sva_cache_set_workspace", "sva_attend_nodes_noalloc", "sva_poll_device_status",
             "sva_debug_inject", "sva_destroy", "sva_last_error")
@@ -98,6 +99,7 @@ def load(path: str = LIB_PATH):
         "sva_attend_nodes": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
         "sva_attend_nodes_sparse": ([p, pn, i32, p, p, p, ctypes.c_float, p, i32, p], i32),
         "sva_qkv_project": ([p, p, i32, i32, p, p, p, p, p, p], i32),
+        "sva_qkv_project_rope": ([p, pn, i32, p, i32, p, p, p, p], i32),
         "sva_attend_nodes_masked": ([p, pn, i32, p, p, p, ctypes.c_float, p, p], i32),
         "sva_attend_workspace_bytes": ([p], ctypes.c_size_t),
         "sva_attend_nodes_noalloc": ([p, pn, i32, p, p, p, ctypes.c_float, p], i32),
@@ -376,6 +378,36 @@ class Cache:
                                   ctypes.c_void_p(q.data_ptr()), ctypes.c_void_p(k.data_ptr()),
                                   ctypes.c_void_p(v.data_ptr()),
                                   ctypes.c_void_p(_stream_handle(stream)))
+        _check(st)
+
+    def qkv_project_rope(self, nodes, x, weight, bias, q, stream=None, check=True):
+        """sva_qkv_project_rope: the projection with RoPE and the cache write fused
+        into its epilogue.  x [n][T][C] bf16 (node i's token rows), weight and
+        bias as qkv_project, q [n][T][H][d] bf16 receives Q'; K' and V go to the
+        nodes' own slots."""
+        n = len(nodes) if not isinstance(nodes, ctypes.Array) else None
+        arr = nodes if isinstance(nodes, ctypes.Array) else make_nodes(nodes)
+        count = n if n is not None else len(arr)
+        g = self.g
+        n_out = g.num_heads * g.head_dim
+        C = int(x.shape[-1])
+        if check:
+            for t, nm in ((x, "x"), (weight, "weight"), (q, "q")):
+                if t.dtype != torch.bfloat16 or not t.is_cuda or not t.is_contiguous():
+                    raise ValueError(f"{nm} must be a contiguous bf16 CUDA tensor")
+            if x.numel() != count * self.T * C:
+                raise ValueError(f"x must hold n_nodes * T rows of {C} features")
+            if tuple(weight.shape) != (3 * n_out, C):
+                raise ValueError(f"weight must be [{3 * n_out}][{C}]")
+            _tok_major(q, "q", count, self.T, g.num_heads, g.head_dim)
+            if bias is not None and (bias.dtype != torch.float32 or not bias.is_cuda
+                                     or not bias.is_contiguous() or bias.numel() != 3 * n_out):
+                raise ValueError(f"bias must be a contiguous fp32 CUDA tensor of {3 * n_out}")
+        st = _lib.sva_qkv_project_rope(self.handle, arr, count, ctypes.c_void_p(x.data_ptr()), C,
+                                       ctypes.c_void_p(weight.data_ptr()),
+                                       ctypes.c_void_p(bias.data_ptr() if bias is not None else 0),
+                                       ctypes.c_void_p(q.data_ptr()),
+                                       ctypes.c_void_p(_stream_handle(stream)))
         _check(st)
 
     def workspace_bytes(self) -> int:

@@ -89,7 +89,7 @@ def test_cache_bytes(sva_mod):
     g = sva_mod.make_geometry(12, 128, 3, 30, 52, num_slots=10, pairs=(22, 21, 21), max_frames=66)
     T, Tpad = 4680, 4736
     pool = 10 * 2 * 12 * Tpad * 128 * 2
-    tabs = [66 * 22 * 8, 30 * 21 * 8, 52 * 21 * 8]
+    tabs = [66 * 22 * 8, 30 * 21 * 8, 52 * 21 * 8, 30 * 21 * 8, 52 * 21 * 8]  # + pair-major h, w
     expect = -(-pool // 256) * 256
     for t in tabs:
         expect = -(-(expect + t) // 256) * 256

@@ -106,3 +106,118 @@ def test_projection_argument_errors(sva_mod):
     st = lib.sva_qkv_project(cache.handle, None, 64, 128, p(z), None, p(z), p(z), p(z), None)
     assert st == sva_mod.ERR_INVALID_ARGUMENT
     cache.close()
+
+
+# ---------------------------------------------------------------- fused projection + RoPE + cache write
+
+def _fused(w, C, rows_sample=None):
+    """Runs sva_qkv_project_rope for the workload's nodes; returns the step,
+    the device Q', the host x, weight, bias and the node table."""
+    inp = I.generate(w)
+    dev = torch.device("cuda")
+    step = Step(w)
+    step.prefill(inp)
+    x, wt, b = I.projection_inputs(w, C)
+    nodes, n = step.node_table()
+    q = torch.empty((n, w.T, w.H, w.d), dtype=torch.bfloat16, device=dev)
+    step.cache.qkv_project_rope(nodes, x.to(dev).contiguous(), wt.to(dev).contiguous(), b.to(dev), q)
+    assert step.cache.poll() == 0
+    return step, inp, q, x, wt, b, nodes
+
+
+def _fused_reference(w, x, wt, b, rows_by_node):
+    """Oracle Q', K', V of the requested token rows of each node (fp64):
+    the projection of those rows, placed in a zero [T][H][d] block so that
+    rope_head rotates them at their own positions."""
+    g = P.oracle_geometry(w)
+    C = x.shape[-1]
+    xs = x.double().numpy().reshape(w.n_nodes, w.T, C)
+    ref = []
+    for i, (_, chunk, _) in enumerate(w.nodes):
+        rows = np.asarray(rows_by_node[i])
+        q, k, v = oracle.qkv_project(xs[i, rows], wt.double().numpy(), b.double().numpy(), heads=w.H)
+        full = [np.zeros((w.T, w.H, w.d)) for _ in range(3)]
+        for t, a in zip(full, (q, k, v)):
+            t[rows] = a
+        for h in range(w.H):
+            full[0][:, h] = oracle.rope_head(full[0][:, h], chunk, g)
+            full[1][:, h] = oracle.rope_head(full[1][:, h], chunk, g)
+        ref.append([t[rows] for t in full])
+    return ref
+
+
+def _check_fused(w, step, q, ref, rows_by_node, nodes):
+    pool = step.cache.slot_pool()
+    gq = q.float().cpu().numpy()
+    for i in range(w.n_nodes):
+        rows = np.asarray(rows_by_node[i])
+        slot = nodes[i].own_slot
+        gk = pool[slot, 0, :, : w.T, :].permute(1, 0, 2).float().cpu().numpy()[rows]
+        gv = pool[slot, 1, :, : w.T, :].permute(1, 0, 2).float().cpu().numpy()[rows]
+        _check(gq[i, rows], ref[i][0], f"{w.name} node {i} Q'")
+        _check(gk, ref[i][1], f"{w.name} node {i} K'")
+        _check(gv, ref[i][2], f"{w.name} node {i} V")
+
+
+def test_fused_projection_rope_tiny_all_rows(oracle_mod):
+    w = I.WORKLOADS["tiny"]                     # H*d = 128: 128-wide tiles, 2 nodes
+    step, inp, q, x, wt, b, nodes = _fused(w, 192)
+    rows = [range(w.T)] * w.n_nodes
+    _check_fused(w, step, q, _fused_reference(w, x, wt, b, rows), rows, nodes)
+    step.close()
+
+
+def test_fused_projection_rope_wan_geometry_sampled(oracle_mod):
+    w = I.WORKLOADS["prog4"]                    # 4 nodes x 4680 rows, 1536 -> 3 x 12 x 128
+    step, inp, q, x, wt, b, nodes = _fused(w, 1536)
+    rng = np.random.default_rng(22)
+    rows = [sorted(set(rng.choice(w.T, 60, replace=False).tolist()) | {0, 127, 128, 1559, 1560, w.T - 1})
+            for _ in range(w.n_nodes)]
+    _check_fused(w, step, q, _fused_reference(w, x, wt, b, rows), rows, nodes)
+    step.close()
+
+
+def test_fused_projection_rope_feeds_attention(oracle_mod):
+    """x -> sva_qkv_project_rope -> sva_attend_nodes against the oracle chain
+    (projection rounded to bf16, then node_forward's RoPE): the fused path
+    skips that intermediate rounding, which the attention tolerance covers."""
+    w = I.WORKLOADS["tiny"]
+    C = 128
+    step, inp, q, x, wt, b, nodes = _fused(w, C)
+    out, lse = step.outputs()
+    step.attend(nodes, q, out, lse)
+    assert step.cache.poll() == 0
+    rq, rk, rv = oracle.qkv_project(x.double().numpy().reshape(-1, C), wt.double().numpy(),
+                                    b.double().numpy(), heads=w.H)
+    shape = (w.n_nodes, w.T, w.H, w.d)
+    rq, rk, rv = (torch.from_numpy(oracle.bf16(t).reshape(shape)) for t in (rq, rk, rv))
+    inp2 = I.Inputs(inp.history, rq, rk, rv)
+    states = P.oracle_states(w, inp2)
+    got = out.float().cpu().numpy()
+    for i in range(w.n_nodes):
+        ref, _ = P.oracle_node(w, inp2, states, i, range(w.H), range(w.T))
+        for h in range(w.H):
+            P.assert_close(got[i, :, h, :], ref[h], f"fused chain node {i} head {h}")
+    step.close()
+
+
+def test_fused_projection_rope_argument_errors(sva_mod):
+    w = I.WORKLOADS["tiny"]
+    step = Step(w)
+    step.prefill(I.generate(w))
+    nodes, n = step.node_table()
+    dev = torch.device("cuda")
+    x = torch.zeros((n, w.T, 128), dtype=torch.bfloat16, device=dev)
+    wt = torch.zeros((3 * w.H * w.d, 128), dtype=torch.bfloat16, device=dev)
+    q = torch.empty((n, w.T, w.H, w.d), dtype=torch.bfloat16, device=dev)
+    lib = sva_mod.load()
+    p = lambda t: __import__("ctypes").c_void_p(t.data_ptr())
+    dup = sva_mod.make_nodes([dict(seq=nodes[0].seq, chunk=nodes[0].chunk, level=nodes[0].level,
+                                   own_slot=nodes[0].own_slot, ctx=[])] * 2)
+    assert lib.sva_qkv_project_rope(step.cache.handle, dup, 2, p(x), 128, p(wt), None, p(q),
+                                    None) == sva_mod.ERR_INVALID_ARGUMENT   # the same own slot twice
+    assert lib.sva_qkv_project_rope(step.cache.handle, nodes, n, p(x), 100, p(wt), None, p(q),
+                                    None) == sva_mod.ERR_INVALID_ARGUMENT   # in_features % 8
+    assert lib.sva_qkv_project_rope(step.cache.handle, nodes, 0, p(x), 128, p(wt), None, p(q),
+                                    None) == sva_mod.ERR_INVALID_ARGUMENT   # no node
+    step.close()
