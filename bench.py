@@ -63,7 +63,8 @@ class L2Flush:
         self.r.sum(dtype=self.acc)
 
 def attn_flops(w) -> float:
-    """Algorithmic FLOPs of one step's attention: 4*T*Lkv*d*H per node (QK^T + PV).
+    """Algorithmic FLOPs of one step's attention: 4*T*Lkv*d*H per node (QK^T + PV),
+    counting under frame causality only the visible (query, own key) pairs.
     With a block-sparse mask only the (query tile, key tile) pairs the mask
     keeps count, each as 4 * rows * keys * d * H (ragged last tiles included
     at their true size)."""
@@ -80,9 +81,14 @@ def attn_flops(w) -> float:
                     if keep[i, qt, k]:
                         total += 4.0 * size[qt] * size[k % nt] * w.d * w.H
         return total
+    # own chunk: every key, or under frame causality the keys up to the end
+    # of the query's latent frame
+    ft = w.Hp * w.Wp
+    own = (float(w.T) * w.T if w.within != "frame_causal"
+           else float(sum(ft * min(T_end, w.T) for T_end in range(ft, w.T + ft, ft))))
     for (_, b, _) in w.nodes:
         n_ctx = max(0, min(w.W, b - 1))
-        total += 4.0 * w.T * (1 + n_ctx) * w.T * w.d * w.H
+        total += 4.0 * (own + float(w.T) * n_ctx * w.T) * w.d * w.H
     return total
 
 

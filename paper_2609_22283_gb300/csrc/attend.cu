@@ -197,12 +197,26 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
   const int n_all = nd.n_kv * p.nt_slot;  // key tiles of the node
   const int qt0 = 2 * qp;
   const bool has_q1 = qt0 + 1 < p.n_qt;
-  // Key tiles of this CTA: a contiguous range of the node's tiles, or under
-  // a block-sparse mask a contiguous range of the tiles either query tile
-  // may attend (set in the prologue below).
+  // Under frame causality the own chunk's key tiles past the frame of the
+  // pair's last query row hold no key that either query tile may see: the
+  // node's key tiles [gap_lo, gap_hi) are skipped.
+  int gap_lo = n_all, gap_hi = n_all;
+  if (nd.frame_causal) {
+    const int last_row = min((qt0 + (has_q1 ? 2 : 1)) * kTile, p.T) - 1;
+    const int frame_end = (last_row / p.frame_tokens + 1) * p.frame_tokens;
+    gap_lo = min((frame_end + kTile - 1) / kTile, p.nt_slot);
+    gap_hi = p.nt_slot;
+  }
+  // the key tile after kt in this CTA's walk (dense instances)
+  auto next_kt = [gap_lo, gap_hi](int kt) { return kt + 1 == gap_lo ? gap_hi : kt + 1; };
+  // Key tiles of this CTA: a contiguous range of the node's tiles that are
+  // not skipped, or under a block-sparse mask a contiguous range of the
+  // tiles either query tile may attend (set in the prologue below).
   constexpr bool sparse = kSparse;  // a launch with a block-sparse tile mask
-  int t_begin = (int)((long long)split * n_all / ns);
-  int n_tiles = (int)((long long)(split + 1) * n_all / ns) - t_begin;
+  const int n_eff = n_all - (gap_hi - gap_lo);
+  int t_begin = (int)((long long)split * n_eff / ns);
+  int n_tiles = (int)((long long)(split + 1) * n_eff / ns) - t_begin;
+  if (t_begin >= gap_lo) t_begin += gap_hi - gap_lo;
   // per query tile, bit i = kernel key tile i (block-sparse instances only)
   __shared__ uint32_t tmask[2][kSparse ? kMaskWords : 1];
   __shared__ int sp_first, sp_count;
@@ -243,7 +257,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     for (int w = 0; w < words; ++w) {
       const int i = (w << 5) + lane;
       bool b0 = false, b1 = false;
-      if (i < n_all) {
+      if (i < n_all && (i < gap_lo || i >= gap_hi)) {
         const int s = i / p.nt_slot;
         const int k = nd.src[s] * p.nt_slot + (i - s * p.nt_slot);
         b0 = row0 ? ((row0[k >> 5] >> (k & 31)) & 1u) != 0u : true;
@@ -309,7 +323,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       }
       const uint64_t keep = l2_policy_evict_last();
       int i = t_begin;  // key tile of the node
-      for (int j = 0; j < n_tiles; ++j, i = sparse ? next_tile(tmask, i + 1, n_all) : i + 1) {
+      for (int j = 0; j < n_tiles; ++j, i = sparse ? next_tile(tmask, i + 1, n_all) : next_kt(i)) {
         const int ks = j % C::kKStages;
         const int vs = j % C::kVStages;
         const int slot = nd.slot[i / p.nt_slot];
@@ -415,7 +429,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         for (int i = 0; ok && i < n_tiles; ++i) {
           const uint32_t par = (uint32_t)i & 1u;
           const bool more = i + 1 < n_tiles;
-          const int kt_next = !more ? kt : (sparse ? next_tile(tmask, kt + 1, n_all) : kt + 1);
+          const int kt_next = !more ? kt : (sparse ? next_tile(tmask, kt + 1, n_all) : next_kt(kt));
           // V_i and K_{i+1} normally land before the softmax hands over P_b,
           // so their waits go first, off the path from P_b to the next MMA.
           if (!wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u) ||
@@ -503,7 +517,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     const bool releaser = warp == 4 && lane == 0;
     bool ok = true;
     int kt = t_begin;  // key tile of the node
-    for (int i = 0; ok && i < n_tiles; ++i, kt = sparse ? next_tile(tmask, kt + 1, n_all) : kt + 1) {
+    for (int i = 0; ok && i < n_tiles; ++i, kt = sparse ? next_tile(tmask, kt + 1, n_all) : next_kt(kt)) {
       const int t = kt % p.nt_slot;  // key tile inside its slot
       const int valid_tile = (t == p.nt_slot - 1) ? p.valid_last : kTile;
       const bool own_fc = frame_causal && kt < p.nt_slot;
@@ -658,7 +672,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
 #pragma unroll
           for (int c = 0; c < DH / 32; ++c) {
             uint32_t o[32];
-            if (!sparse || o_has[b]) {  // dense ranges are never empty
+            if (sparse ? o_has[b] : n_tiles > 0) {  // some key tile was attended
               tmem_ld16x2_32<DH>(tbase + lane_off + col_o(b) + c * 32, o);
               tmem_wait_ld(o);
             } else {  // no key tile attended in this range (block-sparse): no MMA wrote O
@@ -699,7 +713,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
 #pragma unroll
           for (int c = 0; c < DH / 32; ++c) {
             uint32_t o[32];
-            if (!sparse || o_has[b]) {  // dense ranges are never empty
+            if (sparse ? o_has[b] : n_tiles > 0) {  // some key tile was attended
               tmem_ld16x2_32<DH>(tbase + lane_off + col_o(b) + c * 32, o);
               tmem_wait_ld(o);
             } else {  // no key tile attended in this range (block-sparse): no MMA wrote O

@@ -258,6 +258,20 @@ size_t ws_total_bytes(const sva_cache* c) {
 // Splits per work unit: the smallest s in 1..kMaxSplit minimising the wave
 // count per split, ceil(units * s / SMs) / s, subject to the workspace
 // capacity and to at least 4 key tiles per split.
+// Fewest key tiles a work unit of node i walks: all of its slots' tiles,
+// except under frame causality, where a pair of query tiles skips the own
+// chunk's tiles past its last row's frame (the first pair skips the most).
+int key_tiles_walked(const sva_cache* c, const sva::AttnNode& n, int nt_slot) {
+  int own = nt_slot;
+  if (n.frame_causal) {
+    const int frame_tokens = c->g.grid_h * c->g.grid_w;
+    const int last_row = std::min(2 * sva::kTile, c->L.T) - 1;
+    const int frame_end = (last_row / frame_tokens + 1) * frame_tokens;
+    own = std::min((frame_end + sva::kTile - 1) / sva::kTile, nt_slot);
+  }
+  return (n.n_kv - 1) * nt_slot + own;
+}
+
 int choose_split(const sva_cache* c, long long units, int min_tiles) {
   if (c->ws == nullptr) return 1;
   const long long sms = c->num_sms;
@@ -714,7 +728,8 @@ sva_status attend(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const vo
   p.timeout_ns = c->timeout_ns;
   c->fault_mode = 0;
   int min_tiles = 1 << 30;
-  for (int i = 0; i < n_nodes; ++i) min_tiles = std::min(min_tiles, p.nodes[i].n_kv * p.nt_slot);
+  for (int i = 0; i < n_nodes; ++i)
+    min_tiles = std::min(min_tiles, key_tiles_walked(c, p.nodes[i], p.nt_slot));
   const long long units = (long long)g.num_heads * n_nodes * p.n_qp;
   long long n_full = 0;
   int n_split = 1;
@@ -948,7 +963,8 @@ sva_status sva_attend_nodes_noalloc(sva_cache* c, const sva_node* nodes, int32_t
   p.n_qp = (p.n_qt + 1) / 2;
   p.nt_slot = c->L.Tpad / sva::kTile;
   int min_tiles = 1 << 30;
-  for (int i = 0; i < n_nodes; ++i) min_tiles = std::min(min_tiles, p.nodes[i].n_kv * p.nt_slot);
+  for (int i = 0; i < n_nodes; ++i)
+    min_tiles = std::min(min_tiles, key_tiles_walked(c, p.nodes[i], p.nt_slot));
   const long long units = (long long)g.num_heads * n_nodes * p.n_qp;
 
   // The split plan a full workspace would get; its scratch must fit the array.

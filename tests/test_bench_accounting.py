@@ -27,3 +27,16 @@ def test_sparse_counts():
     own_only = sum(4.0 * dense.T * dense.T * dense.d * dense.H for _ in dense.nodes)
     assert bench.attn_flops(none) == own_only
     assert own_only < bench.attn_flops(dense) < bench.attn_flops(base)
+
+
+def test_frame_causal_counts():
+    # prog4fc: 3 frames of 1560 tokens; a query of frame f sees 1560 (f + 1)
+    # own keys, so the own chunk holds 1560^2 (1 + 2 + 3) visible pairs
+    w = I.WORKLOADS["prog4fc"]
+    own = 1560.0 * 1560 * 6
+    assert bench.attn_flops(w) == 4 * 4.0 * (own + 4680.0 * 6 * 4680) * 128 * 12
+    # frame boundaries inside a 128-token tile are counted at token precision
+    t = I.WORKLOADS["tinyfc"]                   # 3 frames of 32 tokens, T = 96
+    per_node = [4.0 * (32 * (32 + 64 + 96) + 96 * max(0, min(t.W, b - 1)) * 96) * t.d * t.H
+                for (_, b, _) in t.nodes]
+    assert bench.attn_flops(t) == sum(per_node)
