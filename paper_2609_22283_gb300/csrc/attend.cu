@@ -146,28 +146,45 @@ struct Bars {
   uint64_t v_empty[4];
 };
 
-// Block-sparse launches: the first key tile at or after `from` that either
-// query tile of the unit may attend (bitmaps in the kernel's tile order), or
-// n_all if there is none.
+// Block-sparse launches: a role's walk over the key tiles that either query
+// tile of the unit may attend (bitmaps in the kernel's tile order).  The
+// current word's remaining bits stay in a register, so a step reads shared
+// memory only when it moves to the next word.  start() takes a set bit (or
+// n_all); the first next() returns it, each later one the following tile of
+// the walk, or n_all past the last.
 template <int W>
-__device__ __forceinline__ int next_tile(const uint32_t (*tm)[W], int from, int n_all) {
-  if (from >= n_all) return n_all;
-  const int words = (n_all + 31) >> 5;
-  int w = from >> 5;
-  uint32_t u = (tm[0][w] | tm[1][w]) & (~0u << (from & 31));
-  while (u == 0) {
-    if (++w >= words) return n_all;
-    u = tm[0][w] | tm[1][w];
+struct TileWalk {
+  const uint32_t (*tm)[W];
+  int n_all, w;
+  uint32_t u;
+  __device__ __forceinline__ void start(const uint32_t (*tm_)[W], int from, int n_all_) {
+    tm = tm_;
+    n_all = n_all_;
+    w = from >> 5;
+    u = from < n_all ? (tm[0][w] | tm[1][w]) & (~0u << (from & 31)) : 0u;
   }
-  return (w << 5) + __ffs(u) - 1;
-}
+  __device__ __forceinline__ int next() {
+    const int words = (n_all + 31) >> 5;
+    while (u == 0u) {
+      if (++w >= words) return n_all;
+      u = tm[0][w] | tm[1][w];
+    }
+    const int k = (w << 5) + __ffs(u) - 1;
+    u &= u - 1u;
+    return k;
+  }
+};
 
 __device__ __forceinline__ void record_timeout(const AttnParams& p, volatile int* abort_flag) {
   *abort_flag = 1;
   atomicCAS(p.status, kStatusOk, kStatusTimeout);
 }
 
-template <int D, bool kSparse>
+// Instances: kSparse = a block-sparse tile mask is walked (all ones when the
+// caller gives none); kOwn = a token-level mask inside the own chunk is
+// applied (only with kSparse).  Each extra feature costs the per-tile loop,
+// so a launch takes the leanest instance that covers it.
+template <int D, bool kSparse, bool kOwn>
 __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_constant__ AttnParams p) {
   using C = AttnCfg<D>;
   extern __shared__ uint8_t smem_raw[];
@@ -322,8 +339,10 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
                       (qt0 + 1) * kTile, nd.q_index);
       }
       const uint64_t keep = l2_policy_evict_last();
-      int i = t_begin;  // key tile of the node
-      for (int j = 0; j < n_tiles; ++j, i = sparse ? next_tile(tmask, i + 1, n_all) : next_kt(i)) {
+      TileWalk<kSparse ? kMaskWords : 1> walk;
+      if constexpr (sparse) walk.start(tmask, t_begin, n_all);
+      int i = sparse ? walk.next() : t_begin;  // key tile of the node
+      for (int j = 0; j < n_tiles; ++j, i = sparse ? walk.next() : next_kt(i)) {
         const int ks = j % C::kKStages;
         const int vs = j % C::kVStages;
         const int slot = nd.slot[i / p.nt_slot];
@@ -418,7 +437,9 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       const int bq = warp == 1 ? 0 : 1;  // the query tile this warp issues for
       bool ok = wait(&bars.q_full, 0);
       if (bq == 0 || has_q1) {
-        int kt = t_begin;  // key tile of the node at iteration i
+        TileWalk<kSparse ? kMaskWords : 1> walk;
+        if constexpr (sparse) walk.start(tmask, t_begin, n_all);
+        int kt = sparse ? walk.next() : t_begin;  // key tile of the node at iteration i
         if (n_tiles > 0) {  // a block-sparse range may be empty: then only o_final is committed
           ok = ok && wait_k(0);
           if (ok) {
@@ -429,7 +450,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         for (int i = 0; ok && i < n_tiles; ++i) {
           const uint32_t par = (uint32_t)i & 1u;
           const bool more = i + 1 < n_tiles;
-          const int kt_next = !more ? kt : (sparse ? next_tile(tmask, kt + 1, n_all) : next_kt(kt));
+          const int kt_next = !more ? kt : (sparse ? walk.next() : next_kt(kt));
+          const bool vis_cur = vis(bq, kt), vis_next = more && vis(bq, kt_next);
           // V_i and K_{i+1} normally land before the softmax hands over P_b,
           // so their waits go first, off the path from P_b to the next MMA.
           if (!wait(&bars.v_full[i % C::kVStages], (uint32_t)(i / C::kVStages) & 1u) ||
@@ -438,8 +460,8 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
             break;
           }
           tc_fence_after();
-          if (vis(bq, kt)) issue_pv(bq, i);
-          if (more) issue_s(bq, i + 1, vis(bq, kt_next));
+          if (vis_cur) issue_pv(bq, i);
+          if (more) issue_s(bq, i + 1, vis_next);
           kt = kt_next;
         }
       }
@@ -516,8 +538,18 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
     // as long as an MMA).
     const bool releaser = warp == 4 && lane == 0;
     bool ok = true;
-    int kt = t_begin;  // key tile of the node
-    for (int i = 0; ok && i < n_tiles; ++i, kt = sparse ? next_tile(tmask, kt + 1, n_all) : next_kt(kt)) {
+    TileWalk<kSparse ? kMaskWords : 1> walk;
+    if constexpr (sparse) walk.start(tmask, t_begin, n_all);
+    int kt = sparse ? walk.next() : t_begin;  // key tile of the node
+    int kt_next = kt;
+    for (int i = 0; ok && i < n_tiles; ++i, kt = kt_next) {
+      // The next tile of the walk and, under a tile mask, which query tiles
+      // attend this one: read from shared memory before the S wait, so their
+      // latency is not added to the path from S to P.
+      kt_next = sparse ? walk.next() : next_kt(kt);
+      const uint32_t attends = sparse ? ((tmask[0][kt >> 5] >> (kt & 31)) & 1u) |
+                                            (((tmask[1][kt >> 5] >> (kt & 31)) & 1u) << 1)
+                                      : 3u;
       const int t = kt % p.nt_slot;  // key tile inside its slot
       const int valid_tile = (t == p.nt_slot - 1) ? p.valid_last : kTile;
       const bool own_fc = frame_causal && kt < p.nt_slot;
@@ -526,7 +558,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
         if (b == 1 && !has_q1) break;
         // own-chunk token mask (masked instance): this thread's 64 bits of its
         // row, fetched before the wait so that the load hides behind it
-        const bool own_tile = sparse && p.own_mask != nullptr && kt < p.nt_slot;
+        const bool own_tile = kOwn && kt < p.nt_slot;
         uint32_t ow[2] = {~0u, ~0u};
         if (own_tile) {
           const int u = (qt0 + b) * kTile + row;
@@ -544,7 +576,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
           mbar_arrive(&bars.k_empty[i % C::kKStages]);
           if (i > 0) mbar_arrive(&bars.v_empty[(i - 1) % C::kVStages]);
         }
-        if (sparse && !((tmask[b][kt >> 5] >> (kt & 31)) & 1u)) {
+        if (sparse && !((attends >> b) & 1u)) {
           // query tile b skips this key tile: no S was computed, no P is due
           mbar_arrive(&bars.p_full[b]);
           continue;
@@ -819,14 +851,16 @@ cudaError_t launch_d(const AttnParams& p, int grid, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (!configured[dev]) {
-    for (auto k : {attend_kernel<D, false>, attend_kernel<D, true>}) {
+    for (auto k : {attend_kernel<D, false, false>, attend_kernel<D, true, false>,
+                   attend_kernel<D, true, true>}) {
       e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
       if (e != cudaSuccess) return e;
     }
     // setmaxnreg.inc waits until the block's register pool can serve it: a
     // build whose launch register count leaves the split short would never
     // proceed, so such a build is refused here.
-    for (auto k : {attend_kernel<D, false>, attend_kernel<D, true>}) {
+    for (auto k : {attend_kernel<D, false, false>, attend_kernel<D, true, false>,
+                   attend_kernel<D, true, true>}) {
       cudaFuncAttributes fa;
       e = cudaFuncGetAttributes(&fa, k);
       if (e != cudaSuccess) return e;
@@ -835,10 +869,12 @@ cudaError_t launch_d(const AttnParams& p, int grid, cudaStream_t s) {
     }
     configured[dev] = true;
   }
-  if (p.masked)
-    attend_kernel<D, true><<<grid, kThreads, C::kSmemBytes, s>>>(p);
+  if (p.masked && p.own_mask != nullptr)
+    attend_kernel<D, true, true><<<grid, kThreads, C::kSmemBytes, s>>>(p);
+  else if (p.masked)
+    attend_kernel<D, true, false><<<grid, kThreads, C::kSmemBytes, s>>>(p);
   else
-    attend_kernel<D, false><<<grid, kThreads, C::kSmemBytes, s>>>(p);
+    attend_kernel<D, false, false><<<grid, kThreads, C::kSmemBytes, s>>>(p);
   return cudaGetLastError();
 }
 
