@@ -97,17 +97,6 @@ __device__ __forceinline__ void mma_commit_mc_warp(uint64_t* bar, uint16_t mask)
       : "memory");
 }
 
-// (cos, sin) of pair `pi` of a head at position (t, hh, ww): pairs [0, P0)
-// rotate with the frame index, [P0, P0+P1) with the patch row, the rest with
-// the patch column (the same values and split as the RoPE + cache write).
-// Here the patch-row and patch-column tables are the pair-major copies
-// ([pair][position]), so the 32 tokens of a warp read neighbouring entries.
-__device__ __forceinline__ float2 rope_cs(const RopeParams& r, int pi, int t, int hh, int ww) {
-  if (pi < r.P0) return __ldg(r.tab_t + (size_t)t * r.P0 + pi);
-  if (pi < r.P0 + r.P1) return __ldg(r.tab_h + (size_t)(pi - r.P0) * r.Hp + hh);
-  return __ldg(r.tab_w + (size_t)(pi - r.P0 - r.P1) * r.Wp + ww);
-}
-
 __device__ __forceinline__ uint32_t rotate2_bf16(float x, float y, float2 cs) {
   const float rx = __fmaf_rn(x, cs.x, -(y * cs.y));
   const float ry = __fmaf_rn(x, cs.y, y * cs.x);
@@ -292,16 +281,35 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
       };
       if (p.rope_on) {
         // Fused RoPE: the 32-column chunk ci of every head in the tile uses
-        // the same 16 (cos, sin) pairs, fetched once.
+        // the same 16 (cos, sin) pairs, fetched once and one chunk ahead.
+        // Pairs [0, P0) rotate with the frame index, [P0, P0+P1) with the
+        // patch row, the rest with the patch column (the values and split of
+        // the RoPE + cache write); the patch-row and patch-column tables
+        // here are the pair-major copies, so the 32 tokens of a warp read
+        // neighbouring entries.
         const RopeParams& rp = p.rope;
         const int cpd = rp.d / 32;  // chunks per head
+        const float2* pt = rp.tab_t + (size_t)tpos * rp.P0;
+
+        auto load_cs = [&](int ci, float2 (&cs)[16]) {
+#pragma unroll
+          for (int e = 0; e < 16; ++e) {
+            const int pi = ci * 16 + e;
+            const float2* a =
+                pi < rp.P0 ? pt + pi
+                           : (pi < rp.P0 + rp.P1 ? rp.tab_h + (size_t)(pi - rp.P0) * rp.Hp + hh
+                                                 : rp.tab_w + (size_t)(pi - rp.P0 - rp.P1) * rp.Wp + ww);
+            cs[e] = __ldg(a);
+          }
+        };
+        float2 cs_next[16];
+        if (tensor != 2) load_cs(0, cs_next);
 #pragma unroll 1
         for (int ci = 0; ci < cpd; ++ci) {
           float2 cs[16];
-          if (tensor != 2) {
 #pragma unroll
-            for (int e = 0; e < 16; ++e) cs[e] = rope_cs(rp, ci * 16 + e, tpos, hh, ww);
-          }
+          for (int e = 0; e < 16; ++e) cs[e] = cs_next[e];
+          if (tensor != 2 && ci + 1 < cpd) load_cs(ci + 1, cs_next);
 #pragma unroll 1
           for (int hb = 0; hb < BN / rp.d; ++hb) {
             const int c = hb * cpd + ci;
