@@ -289,8 +289,7 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
         // neighbouring entries.
         const RopeParams& rp = p.rope;
         const int cpd = rp.d / 32;  // chunks per head
-        const float2* pt = rp.tab_t + (size_t)tpos * rp.P0;
-
+        const float2* pt = rp.tab_t + (size_t)tpos * rp.P0;  // this token's frame row
         auto load_cs = [&](int ci, float2 (&cs)[16]) {
 #pragma unroll
           for (int e = 0; e < 16; ++e) {
