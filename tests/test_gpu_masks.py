@@ -42,6 +42,17 @@ SPLITFC_WARP = I.Workload(name="splitfcwarp", seed=18, F=10, Hp=10, Wp=10, H=1, 
                           within="frame_causal", description="masked and visible rows in one warp")
 
 
+# The first chunk of a video: no history, T = 1024 in four frames of 256
+# tokens, two heads.  The first unit walks only the own chunk's tiles 0-1.
+FC_FIRST = I.Workload(name="fcfirst", seed=19, F=4, Hp=16, Wp=16, H=2, d=128, K=2, W=2,
+                      policy="prog", nodes=((0, 1, 1),), prefilled=(),
+                      within="frame_causal", description="frame-causal node without history")
+
+
+def test_frame_causal_node_without_history(oracle_mod):
+    _all_rows(oracle_mod, FC_FIRST)
+
+
 def test_tiny_frame_causal_all_rows(oracle_mod):
     _all_rows(oracle_mod, I.WORKLOADS["tinyfc"])
 
