@@ -70,8 +70,9 @@ struct AttnCfg {
 __device__ __forceinline__ uint32_t col_s(int b) { return b ? 128u : 0u; }
 __device__ __forceinline__ uint32_t col_o(int b) { return b ? 384u : 256u; }
 
-// 12 warps: warpgroup 0 = TMA producer (warp 0), MMA issuer (warp 1), two
-// idle warps; warpgroups 1 and 2 = softmax.  The launch gives every thread
+// 12 warps: warpgroup 0 = TMA producer (warp 0), MMA issuers (warps 1 and
+// 3), warp 2 (the block-sparse mask gather in the prologue, then idle);
+// warpgroups 1 and 2 = softmax.  The launch gives every thread
 // kLaunchRegs registers; warpgroup 0 then gives registers back
 // (setmaxnreg.dec to kRegsLow) and the softmax warpgroups take them
 // (setmaxnreg.inc to kRegsHigh).  The split must fit the launch's pool:
@@ -480,7 +481,7 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
       // Some wait expired.  Before the CTA exits, wait (bounded, ignoring
       // the abort flag) for what this CTA still has in flight: the TMA
       // copies the producer started (a stage's barrier cannot run ahead of
-      // the last copy started into it) and every MMA the issuer started.
+      // the last copy started into it) and every MMA the issuers started.
       const int zero = 0;
       if (warp == 0 && lane == 0) {
         mbar_wait(&bars.q_full, 0, &zero, tmo);
