@@ -97,10 +97,17 @@ def rope_bytes(w) -> float:
 
 
 def kernel_hash() -> str:
+    """Hash of the attention kernel's code: its sources with comments and
+    whitespace removed, so that a comment edit keeps the ncu counters valid
+    and any change to the code voids them."""
+    import re
     h = hashlib.sha256()
     for f in KERNEL_SOURCES:
-        with open(os.path.join(ROOT, f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, f), encoding="utf-8") as fh:
+            src = fh.read()
+        src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+        src = re.sub(r"//[^\n]*", " ", src)
+        h.update("".join(src.split()).encode())
     return h.hexdigest()[:16]
 
 
