@@ -167,6 +167,18 @@ def test_fused_projection_rope_tiny_all_rows(oracle_mod):
     step.close()
 
 
+def test_fused_projection_rope_four_heads_per_tile(oracle_mod):
+    # H*d = 256 with d = 64: 256-wide tiles holding four heads, 3 latent
+    # frames of 6 x 10 tokens (T = 180, ragged last 128-row tile)
+    base = I.WORKLOADS["tiny"]
+    w = I.Workload(**{**base.__dict__, "name": "tinyh4", "F": 3, "Hp": 6, "Wp": 10, "H": 4,
+                      "pairs": None})
+    step, inp, q, x, wt, b, nodes = _fused(w, 96)
+    rows = [range(w.T)] * w.n_nodes
+    _check_fused(w, step, q, _fused_reference(w, x, wt, b, rows), rows, nodes)
+    step.close()
+
+
 def test_fused_projection_rope_wan_geometry_sampled(oracle_mod):
     w = I.WORKLOADS["prog4"]                    # 4 nodes x 4680 rows, 1536 -> 3 x 12 x 128
     step, inp, q, x, wt, b, nodes = _fused(w, 1536)
