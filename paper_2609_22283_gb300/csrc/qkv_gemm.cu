@@ -8,24 +8,30 @@
 //   N = H*d is not a multiple of 256), 64-wide K blocks through a 4-stage
 //   TMA ring.
 //
-// Persistent CTAs (one per SM) walk the output tiles; two TMEM accumulators
-// let the epilogue of one tile (TMEM -> + bias -> bf16 -> global) overlap the
-// main loop of the next.  CTAs run in clusters of two that take vertically
-// adjacent tiles (same W rows): each loads its own x tile and half of the W
-// tile, multicast into both CTAs' shared memory, so a CTA pulls 32 KB per K
-// block from L2 instead of 48 KB (the 4-stage ring holds too little to hide
-// the L2 latency at 48 KB per 512 MMA cycles).
-//   warp 0     TMA producer (x and W tiles, 128-byte swizzle);
-//   warp 1     TMEM owner and MMA issuer (whole warp, one elected lane);
-//   warps 4-7  epilogue, one output row per thread.
-// A tile never straddles q, k and v (N is a multiple of BN), so its epilogue
+// Persistent CTAs (one per SM) walk a list of work items; two TMEM
+// accumulators let the epilogue of one item (TMEM -> + bias -> bf16 ->
+// global) overlap the main loop of the next.  Items are output tiles with
+// the column tile varying fastest, so the CTAs running at one time read the
+// same few x row tiles (shared through L2) and all of W (which stays in L2).
+// When the tiles do not fill the last round of CTAs, the tiles of that round
+// are split into two half-width items (BN / 2 columns), so that the last
+// round takes half as long.
+//   warp 0      TMA producer (x and W tiles, 128-byte swizzle);
+//   warp 1      TMEM owner and MMA issuer (whole warp, one elected lane);
+//   warps 4-11  epilogue: two warps per TMEM lane quarter, one output row per
+//               thread, the two warps of a quarter taking alternate 32-column
+//               chunks.
+// An item never straddles q, k and v (N is a multiple of BN), so its epilogue
 // writes into one tensor.  With the fused RoPE epilogue (sva_qkv_project_rope)
 // each thread rotates the pairs of its row's q and k columns in fp32 at the
 // token's (t, h, w) position before the one bf16 rounding, writes Q' token-
-// major and scatters K' and V into the node's own cache slot.  Rows past `rows` read zeros (TMA fill) and are
-// not stored; K past C reads zeros on both operands.  All waits are bounded:
-// on expiry the CTA records SVA_ERR_DEVICE_TIMEOUT, drains its own copies and
-// MMAs, frees TMEM and exits.
+// major and scatters K' and V into the node's own cache slot.  Rows past
+// `rows` read zeros (TMA fill) and are not stored; K past C reads zeros on
+// both operands.  All waits are bounded: on expiry the CTA records
+// SVA_ERR_DEVICE_TIMEOUT, drains its own copies and MMAs, frees TMEM and
+// exits.
+#include <mutex>
+
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -37,10 +43,11 @@ namespace {
 
 using namespace ptx;
 
-constexpr int kProjThreads = 256;
+constexpr int kProjThreads = 384;
 constexpr int kStages = 4;
 constexpr int kBM = 128;
 constexpr int kBK = 64;
+constexpr int kEpiWarps = 8;
 
 template <int BN>
 struct ProjCfg {
@@ -53,48 +60,15 @@ struct ProjCfg {
 
 struct ProjBars {
   uint64_t full[kStages];
-  uint64_t empty[kStages];  // both CTAs' MMAs have read the stage (two arrivals)
+  uint64_t empty[kStages];
   uint64_t acc_full[2];
-  uint64_t acc_empty[2];
+  uint64_t acc_empty[2];  // one arrival per epilogue warp
   uint64_t drain;
 };
 
 __device__ __forceinline__ uint32_t pack2_bf16(float lo, float hi) {
   __nv_bfloat162 r = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&r);
-}
-
-__device__ __forceinline__ uint32_t cluster_rank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
-// TMA 2D tile load written to the same offset of every CTA in `mask`, each
-// CTA's barrier at `bar`'s offset receiving the completed bytes.
-__device__ __forceinline__ void tma_load_2d_mc(void* dst, const CUtensorMap* map, uint64_t* bar,
-                                               int32_t c0, int32_t c1, uint16_t mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
-      " [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(smem_u32(bar)), "r"(c0), "r"(c1), "h"(mask)
-      : "memory");
-}
-
-// Arrives on the barrier at `bar`'s offset in every CTA of `mask` once this
-// thread's MMAs so far have completed (one elected lane of a converged warp).
-__device__ __forceinline__ void mma_commit_mc_warp(uint64_t* bar, uint16_t mask) {
-  asm volatile(
-      "{\n"
-      " .reg .pred e;\n"
-      " elect.sync _|e, 0xffffffff;\n"
-      " @e tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;\n"
-      "}\n" ::"r"(smem_u32(bar)), "h"(mask)
-      : "memory");
 }
 
 __device__ __forceinline__ uint32_t rotate2_bf16(float x, float y, float2 cs) {
@@ -106,6 +80,25 @@ __device__ __forceinline__ uint32_t rotate2_bf16(float x, float y, float2 cs) {
 __device__ __forceinline__ void proj_timeout(const ProjParams& p, volatile int* abort_flag) {
   *abort_flag = 1;
   atomicCAS(p.status, kStatusOk, kStatusTimeout);
+}
+
+// Work item i: output tile (m, n), whole (half = -1) or its column half
+// `half` (items past n_whole, two per tile).
+struct Item {
+  int m, n, half;
+};
+
+__device__ __forceinline__ Item item_of(const ProjParams& p, int i) {
+  Item it;
+  int t = i;
+  it.half = -1;
+  if (i >= p.n_whole) {
+    t = p.n_whole + ((i - p.n_whole) >> 1);
+    it.half = (i - p.n_whole) & 1;
+  }
+  it.m = t / p.n_ntiles;
+  it.n = t - it.m * p.n_ntiles;
+  return it;
 }
 
 template <int BN>
@@ -120,22 +113,16 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  // pairs of tiles (m pair, n): cluster c takes pairs c, c + clusters, ...;
-  // CTA `rank` of the cluster computes m tile 2 * m_pair + rank
-  const uint32_t rank = cluster_rank();
-  const int cluster = blockIdx.x >> 1, clusters = gridDim.x >> 1;
-  const int n_mpairs = (p.n_mtiles + 1) >> 1;
-  const int total = n_mpairs * p.n_ntiles;
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
     for (int s = 0; s < kStages; ++s) {
       mbar_init(&bars.full[s], 1);
-      mbar_init(&bars.empty[s], 2);
+      mbar_init(&bars.empty[s], 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bars.acc_full[b], 1);
-      mbar_init(&bars.acc_empty[b], 128);
+      mbar_init(&bars.acc_empty[b], kEpiWarps);
     }
     mbar_init(&bars.drain, 1);
     fence_mbar_init();
@@ -146,7 +133,6 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
   }
   tc_fence_before();
   __syncthreads();
-  cluster_sync();  // both CTAs' barriers are initialised before either multicasts
   tc_fence_after();
   const uint32_t tbase = tmem_base_sh;
   const uint64_t tmo = p.timeout_ns;
@@ -157,10 +143,13 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
     if (lane == 0) {
       prefetch_tmap(&p.tmap_x);
       prefetch_tmap(&p.tmap_w);
-      bool ok = true;
-      for (int t = cluster; ok && t < total; t += clusters) {
-        const int mp = t / p.n_ntiles, n = t - (t / p.n_ntiles) * p.n_ntiles;
-        const int m = 2 * mp + (int)rank;  // past the last m tile: rows read as zeros
+      prefetch_tmap(&p.tmap_wh);
+      for (int i = blockIdx.x; i < p.n_items; i += gridDim.x) {
+        const Item it = item_of(p, i);
+        const bool half = it.half >= 0;
+        const uint32_t bytes = C::kABytes + (half ? C::kBBytes / 2 : C::kBBytes);
+        const int w_row = it.n * BN + (half ? it.half * (BN / 2) : 0);
+        bool ok = true;
         for (int kb = 0; kb < p.n_kblocks; ++kb, ++issued) {
           const int s = issued % kStages;
           const uint32_t ph = (uint32_t)(issued / kStages) & 1u;
@@ -170,26 +159,18 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
             break;
           }
           uint8_t* sa = smem + s * C::kStageBytes;
-          mbar_arrive_expect_tx(&bars.full[s], C::kStageBytes);
-          tma_load_2d(sa, &p.tmap_x, &bars.full[s], kb * kBK, m * kBM);
-          // this CTA's half of the W tile, into both CTAs
-          tma_load_2d_mc(sa + C::kABytes + rank * (C::kBBytes / 2), &p.tmap_w, &bars.full[s],
-                         kb * kBK, n * BN + (int)rank * (BN / 2), 0x3);
+          mbar_arrive_expect_tx(&bars.full[s], bytes);
+          tma_load_2d(sa, &p.tmap_x, &bars.full[s], kb * kBK, it.m * kBM);
+          tma_load_2d(sa + C::kABytes, half ? &p.tmap_wh : &p.tmap_w, &bars.full[s], kb * kBK,
+                      w_row);
         }
-      }
-      // Every stage must be released by both CTAs' MMAs before this CTA may
-      // leave: the peer's commits arrive on this CTA's empty barriers.
-      for (int j = issued; ok && j < issued + kStages; ++j) {
-        if (!mbar_wait(&bars.empty[j % kStages], ((uint32_t)(j / kStages) & 1u) ^ 1u, &abort_flag,
-                       tmo)) {
-          proj_timeout(p, &abort_flag);
-          ok = false;
-        }
+        if (!ok) break;
       }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    constexpr uint32_t idesc = idesc_bf16_f32(kBM, BN, false);
+    constexpr uint32_t idesc_whole = idesc_bf16_f32(kBM, BN, false);
+    constexpr uint32_t idesc_half = idesc_bf16_f32(kBM, BN / 2, false);
     const uint64_t dA = sdesc_sw128(smem_u32(smem), 16, 1024);
     const uint64_t dB = sdesc_sw128(smem_u32(smem + C::kABytes), 16, 1024);
     constexpr uint64_t kStageStep = (uint64_t)(C::kStageBytes >> 4);
@@ -197,8 +178,9 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
       return __all_sync(0xffffffffu, mbar_wait(bar, parity, &abort_flag, tmo));
     };
     bool ok = true;
-    int it = 0, tc = 0;
-    for (int t = cluster; ok && t < total; t += clusters, ++tc) {
+    int k_it = 0, tc = 0;
+    for (int i = blockIdx.x; ok && i < p.n_items; i += gridDim.x, ++tc) {
+      const uint32_t idesc = item_of(p, i).half >= 0 ? idesc_half : idesc_whole;
       const int acc = tc & 1;
       if (!wait(&bars.acc_empty[acc], ((uint32_t)(tc >> 1) & 1u) ^ 1u)) {
         ok = false;
@@ -206,9 +188,9 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
       }
       tc_fence_after();
       const uint32_t dcol = tbase + (uint32_t)(acc * BN);
-      for (int kb = 0; kb < p.n_kblocks; ++kb, ++it) {
-        const int s = it % kStages;
-        if (!wait(&bars.full[s], (uint32_t)(it / kStages) & 1u)) {
+      for (int kb = 0; kb < p.n_kblocks; ++kb, ++k_it) {
+        const int s = k_it % kStages;
+        if (!wait(&bars.full[s], (uint32_t)(k_it / kStages) & 1u)) {
           ok = false;
           break;
         }
@@ -219,9 +201,7 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
         for (int kk = 0; kk < kBK / 16; ++kk)  // 32 bytes of K per MMA inside the swizzle atom
           mma_ss_warp(dcol, a + (uint64_t)(kk * 2), b + (uint64_t)(kk * 2), idesc,
                       (kb > 0 || kk > 0) ? 1u : 0u);
-        // the stage is free (in both CTAs: half of it came from the peer) once
-        // these MMAs have read it
-        mma_commit_mc_warp(&bars.empty[s], 0x3);
+        mma_commit_warp(&bars.empty[s]);  // the stage is free once these MMAs have read it
       }
       if (!ok) break;
       mma_commit_warp(&bars.acc_full[acc]);
@@ -229,23 +209,24 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
     if (!ok && lane == 0) proj_timeout(p, &abort_flag);
   } else if (warp >= 4) {
     // ------------------------------------------------------------ epilogue
-    const int q4 = warp & 3;
+    const int q4 = warp & 3;           // TMEM lane quarter this warp may access
+    const int part = (warp - 4) >> 2;  // which alternate 32-column chunks
     const int row = q4 * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
     bool ok = true;
     int tc = 0;
-    for (int t = cluster; ok && t < total; t += clusters, ++tc) {
-      const int mp = t / p.n_ntiles, n = t - (t / p.n_ntiles) * p.n_ntiles;
-      const int m = 2 * mp + (int)rank;
+    for (int i = blockIdx.x; ok && i < p.n_items; i += gridDim.x, ++tc) {
+      const Item it = item_of(p, i);
+      const int width = it.half >= 0 ? BN / 2 : BN;  // output columns of this item
       const int acc = tc & 1;
       ok = mbar_wait(&bars.acc_full[acc], (uint32_t)(tc >> 1) & 1u, &abort_flag, tmo);
       ok = __all_sync(0xffffffffu, ok);
       if (!ok) break;
       tc_fence_after();
-      const int col = n * BN;            // output column in [0, 3N)
+      const int col = it.n * BN + (it.half > 0 ? BN / 2 : 0);  // output column in [0, 3N)
       const int tensor = col / p.N;      // q, k or v
       const int c0 = col - tensor * p.N;  // column inside that tensor
-      const long long grow = (long long)m * kBM + row;
+      const long long grow = (long long)it.m * kBM + row;
       const bool in_range = grow < p.rows;
       __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.out[p.rope_on ? 0 : tensor]) + grow * p.N + c0;
       // fused RoPE: this row's node, token and position, and where K' / V go
@@ -280,15 +261,18 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
         }
       };
       if (p.rope_on) {
-        // Fused RoPE: the 32-column chunk ci of every head in the tile uses
-        // the same 16 (cos, sin) pairs, fetched once and one chunk ahead.
-        // Pairs [0, P0) rotate with the frame index, [P0, P0+P1) with the
-        // patch row, the rest with the patch column (the values and split of
-        // the RoPE + cache write); the patch-row and patch-column tables
-        // here are the pair-major copies, so the 32 tokens of a warp read
-        // neighbouring entries.
+        // Fused RoPE: the 32-column chunk ci of every head in the item uses
+        // the same 16 (cos, sin) pairs, fetched once per chunk index (the
+        // next one while the current one is rotated); this warp takes the
+        // chunk indices of its parity.  Pairs [0, P0) rotate with the frame
+        // index, [P0, P0+P1) with the patch row, the rest with the patch
+        // column (the values and split of the RoPE + cache write); the
+        // patch-row and patch-column tables here are the pair-major copies,
+        // so the 32 tokens of a warp read neighbouring entries.  An item
+        // covers whole heads (the host splits a tile only when its halves do).
         const RopeParams& rp = p.rope;
-        const int cpd = rp.d / 32;  // chunks per head
+        const int cpd = rp.d / 32;  // chunks per head (even: d is 64 or 128)
+        const int heads = width / rp.d;
         const float2* pt = rp.tab_t + (size_t)tpos * rp.P0;  // this token's frame row
         auto load_cs = [&](int ci, float2 (&cs)[16]) {
 #pragma unroll
@@ -302,15 +286,15 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
           }
         };
         float2 cs_next[16];
-        if (tensor != 2) load_cs(0, cs_next);
+        if (tensor != 2) load_cs(part, cs_next);
 #pragma unroll 1
-        for (int ci = 0; ci < cpd; ++ci) {
+        for (int ci = part; ci < cpd; ci += 2) {
           float2 cs[16];
 #pragma unroll
           for (int e = 0; e < 16; ++e) cs[e] = cs_next[e];
-          if (tensor != 2 && ci + 1 < cpd) load_cs(ci + 1, cs_next);
+          if (tensor != 2 && ci + 2 < cpd) load_cs(ci + 2, cs_next);
 #pragma unroll 1
-          for (int hb = 0; hb < BN / rp.d; ++hb) {
+          for (int hb = 0; hb < heads; ++hb) {
             const int c = hb * cpd + ci;
             uint32_t r[32];
             float bv[32];
@@ -337,7 +321,7 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
         }
       } else {
 #pragma unroll 1
-        for (int c = 0; c < BN / 32; ++c) {
+        for (int c = part; c < width / 32; c += 2) {
           uint32_t r[32];
           float bv[32];
           load_chunk(c, r, bv);  // warp-collective: every thread, in range or not
@@ -355,8 +339,11 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
           }
         }
       }
+      // The MMA warp may overwrite this accumulator once every epilogue warp
+      // has read its part (each thread waited for its own TMEM loads).
       tc_fence_before();
-      mbar_arrive(&bars.acc_empty[acc]);  // the MMA warp may overwrite this accumulator
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&bars.acc_empty[acc]);
     }
     if (!ok) proj_timeout(p, &abort_flag);
   }
@@ -382,37 +369,35 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
     tc_fence_after();
     tmem_dealloc(tbase, C::kTmemCols);
   }
-  cluster_sync();  // neither CTA leaves while the other may still reach its shared memory
+}
+
+// One-time per-device set-up of a kernel instance (its shared-memory limit),
+// done under a lock so that two host threads launching on the same device
+// for the first time cannot race.
+template <int BN>
+cudaError_t configure_bn(int dev) {
+  using C = ProjCfg<BN>;
+  static std::mutex mu;
+  static bool configured[64] = {};
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (configured[dev]) return cudaSuccess;
+  cudaError_t e = cudaFuncSetAttribute(qkv_project_kernel<BN>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+  if (e != cudaSuccess) return e;
+  configured[dev] = true;
+  return cudaSuccess;
 }
 
 template <int BN>
 cudaError_t launch_bn(const ProjParams& p, int grid, cudaStream_t s) {
   using C = ProjCfg<BN>;
-  static bool configured[64] = {};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if (!configured[dev]) {
-    e = cudaFuncSetAttribute(qkv_project_kernel<BN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             C::kSmemBytes);
-    if (e != cudaSuccess) return e;
-    configured[dev] = true;
-  }
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((unsigned)grid);
-  cfg.blockDim = dim3(kProjThreads);
-  cfg.dynamicSmemBytes = C::kSmemBytes;
-  cfg.stream = s;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 2;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, qkv_project_kernel<BN>, p);
+  e = configure_bn<BN>(dev);
   if (e != cudaSuccess) return e;
+  qkv_project_kernel<BN><<<grid, kProjThreads, C::kSmemBytes, s>>>(p);
   return cudaGetLastError();
 }
 

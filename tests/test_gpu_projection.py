@@ -108,6 +108,52 @@ def test_projection_argument_errors(sva_mod):
     cache.close()
 
 
+@pytest.mark.parametrize("which", ["weight", "x", "bias", "q"])
+def test_projection_rejects_memory_off_the_device(sva_mod, which):
+    """Every operand must be memory of the cache's GPU: a host pointer (here
+    pinned host memory, which the GPU could otherwise reach) is refused with
+    INVALID_ARGUMENT before anything is launched."""
+    import ctypes
+    w = I.WORKLOADS["tiny"]
+    cache = sva.Cache(geometry_for(w))
+    lib = sva_mod.load()
+    dev = torch.device("cuda")
+    rows, C, N = 64, 128, w.H * w.d
+    t = {"x": torch.ones((rows, C), dtype=torch.bfloat16, device=dev),
+         "weight": torch.ones((3 * N, C), dtype=torch.bfloat16, device=dev),
+         "bias": torch.zeros(3 * N, dtype=torch.float32, device=dev),
+         "q": torch.full((rows, N), 7.0, dtype=torch.bfloat16, device=dev)}
+    t[which] = t[which].cpu().pin_memory()
+    k = torch.full((rows, N), 7.0, dtype=torch.bfloat16, device=dev)
+    v = torch.full((rows, N), 7.0, dtype=torch.bfloat16, device=dev)
+    p = lambda a: ctypes.c_void_p(a.data_ptr())
+    st = lib.sva_qkv_project(cache.handle, p(t["x"]), rows, C, p(t["weight"]), p(t["bias"]),
+                             p(t["q"]), p(k), p(v), None)
+    assert st == sva_mod.ERR_INVALID_ARGUMENT, st
+    assert "not device memory" in sva_mod.last_error()
+    torch.cuda.synchronize()
+    assert bool((k == 7.0).all()) and bool((v == 7.0).all())     # nothing was launched
+    assert cache.poll() == 0
+    cache.close()
+
+
+@pytest.mark.parametrize("fused", [False, True])
+def test_projection_three_heads_of_128(oracle_mod, fused):
+    """H*d = 384: 128-wide tiles (one head each).  The plain projection splits
+    its partial last round into 64-wide items; the fused epilogue may not
+    (half a head), so it runs whole tiles.  All rows of 2 nodes of T = 180."""
+    base = I.WORKLOADS["tiny"]
+    w = I.Workload(**{**base.__dict__, "name": "h3d128", "F": 3, "Hp": 6, "Wp": 10, "H": 3,
+                      "d": 128, "pairs": None})
+    if not fused:
+        _project(w, 256)
+        return
+    step, inp, q, x, wt, b, nodes = _fused(w, 256)
+    rows = [range(w.T)] * w.n_nodes
+    _check_fused(w, step, q, _fused_reference(w, x, wt, b, rows), rows, nodes)
+    step.close()
+
+
 # ---------------------------------------------------------------- fused projection + RoPE + cache write
 
 def _fused(w, C, rows_sample=None):
