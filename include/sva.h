@@ -215,8 +215,12 @@ sva_status sva_rope_kv_write_qknorm(sva_cache* c, const sva_node* nodes, int32_t
  *   bias    [3*H*d] fp32, or NULL
  *   q, k, v [rows][H*d] bf16 outputs
  * in_features a positive multiple of 8; H*d a multiple of 128; every pointer
- * 16-byte aligned.  Stream-ordered; a device timeout is reported by
- * sva_poll_device_status.  Errors: INVALID_ARGUMENT, UNSUPPORTED (H*d), CUDA. */
+ * 16-byte aligned and in device memory of the cache's device (a host or
+ * another GPU's pointer is rejected with INVALID_ARGUMENT before anything is
+ * launched).  Each CTA loads its own operand tiles from this GPU's memory
+ * (no copy is shared between CTAs).  Stream-ordered; a device timeout is
+ * reported by sva_poll_device_status.  Errors: INVALID_ARGUMENT,
+ * UNSUPPORTED (H*d), CUDA. */
 sva_status sva_qkv_project(sva_cache* c, const void* x, int32_t rows, int32_t in_features,
                            const void* weight, const float* bias, void* q, void* k, void* v,
                            sva_stream s);
@@ -334,14 +338,16 @@ sva_status sva_cache_set_workspace(sva_cache* c, void* dev_buf, size_t bytes);
  * framework, or a serving loop that forbids cudaMalloc because it can block
  * and synchronise the device.  Such a caller cannot provide the split
  * workspace of sva_cache_set_workspace.  This entry point takes the same
- * arguments and gives the same results (within rounding) as
- * sva_attend_nodes with a workspace attached, but keeps its key-range
- * partials and arrival counters in a scratch array that the library
- * declares in device memory itself (32 MiB, held by every GPU that loads
- * the library until the process exits).  It allocates nothing and calls no
- * allocating routine.  Launches whose split plan needs more than 32 MiB of
- * scratch are rejected with SVA_ERR_CAPACITY and launch nothing; launches
- * that need no split use no scratch and are never rejected for size.
+ * arguments, runs the same checks and chooses the same key-range split plan
+ * as sva_attend_nodes with a workspace attached, so its results are bitwise
+ * the same, but it keeps its key-range partials and arrival counters in a
+ * scratch array that the library declares in device memory itself (32 MiB,
+ * held by every GPU that loads the library until the process exits).  It
+ * allocates nothing and calls no allocating routine.  Launches whose split
+ * plan needs more than 32 MiB of scratch (counters plus 133 KB per split
+ * item at head_dim 128) are rejected with SVA_ERR_CAPACITY and launch
+ * nothing; launches that need no split use no scratch and are never
+ * rejected for size.
  * Each call clears the array's counters on `s` before its kernel; the
  * partials left by one call are overwritten by the next.  All calls on a
  * device share the one array, so calls whose kernels can overlap on the

@@ -39,6 +39,8 @@
 // All waits are bounded (1 s by default): on expiry the CTA records
 // SVA_ERR_DEVICE_TIMEOUT in the status word, drains its own copies and MMAs,
 // frees TMEM and exits.
+#include <mutex>
+
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -843,33 +845,46 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
   }
 }
 
+// One-time per-device set-up of the kernel instances (shared-memory limit,
+// register check), done under a lock so that two host threads launching on
+// the same device for the first time cannot race.
+template <int D>
+cudaError_t configure_d(int dev) {
+  using C = AttnCfg<D>;
+  static std::mutex mu;
+  static bool configured[64] = {};
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (configured[dev]) return cudaSuccess;
+  cudaError_t e;
+  for (auto k : {attend_kernel<D, false, false>, attend_kernel<D, true, false>,
+                 attend_kernel<D, true, true>}) {
+    e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
+    if (e != cudaSuccess) return e;
+  }
+  // setmaxnreg.inc waits until the block's register pool can serve it: a
+  // build whose launch register count leaves the split short would never
+  // proceed, so such a build is refused here.
+  for (auto k : {attend_kernel<D, false, false>, attend_kernel<D, true, false>,
+                 attend_kernel<D, true, true>}) {
+    cudaFuncAttributes fa;
+    e = cudaFuncGetAttributes(&fa, k);
+    if (e != cudaSuccess) return e;
+    if (fa.numRegs * kThreads < 4 * 32 * kRegsLow + 8 * 32 * kRegsHigh)
+      return cudaErrorInvalidConfiguration;
+  }
+  configured[dev] = true;
+  return cudaSuccess;
+}
+
 template <int D>
 cudaError_t launch_d(const AttnParams& p, int grid, cudaStream_t s) {
   using C = AttnCfg<D>;
-  static bool configured[64] = {};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
-  if (!configured[dev]) {
-    for (auto k : {attend_kernel<D, false, false>, attend_kernel<D, true, false>,
-                   attend_kernel<D, true, true>}) {
-      e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes);
-      if (e != cudaSuccess) return e;
-    }
-    // setmaxnreg.inc waits until the block's register pool can serve it: a
-    // build whose launch register count leaves the split short would never
-    // proceed, so such a build is refused here.
-    for (auto k : {attend_kernel<D, false, false>, attend_kernel<D, true, false>,
-                   attend_kernel<D, true, true>}) {
-      cudaFuncAttributes fa;
-      e = cudaFuncGetAttributes(&fa, k);
-      if (e != cudaSuccess) return e;
-      if (fa.numRegs * kThreads < 4 * 32 * kRegsLow + 8 * 32 * kRegsHigh)
-        return cudaErrorInvalidConfiguration;
-    }
-    configured[dev] = true;
-  }
+  e = configure_d<D>(dev);
+  if (e != cudaSuccess) return e;
   if (p.masked && p.own_mask != nullptr)
     attend_kernel<D, true, true><<<grid, kThreads, C::kSmemBytes, s>>>(p);
   else if (p.masked)

@@ -48,6 +48,17 @@ sva_status cuda_fail(cudaError_t e, const char* what) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// True when `p` points into device memory of `device`.
+bool on_device(const void* p, int device) {
+  cudaPointerAttributes attr;
+  const cudaError_t e = cudaPointerGetAttributes(&attr, p);
+  if (e != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return attr.type == cudaMemoryTypeDevice && attr.device == device;
+}
+
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -255,9 +266,6 @@ size_t ws_total_bytes(const sva_cache* c) {
   return ws_counter_bytes(c) + (size_t)ws_items(c) * ws_item_bytes(c);
 }
 
-// Splits per work unit: the smallest s in 1..kMaxSplit minimising the wave
-// count per split, ceil(units * s / SMs) / s, subject to the workspace
-// capacity and to at least 4 key tiles per split.
 // Fewest key tiles a work unit of node i walks: all of its slots' tiles,
 // except under frame causality, where a pair of query tiles skips the own
 // chunk's tiles past its last row's frame (the first pair skips the most).
@@ -272,14 +280,17 @@ int key_tiles_walked(const sva_cache* c, const sva::AttnNode& n, int nt_slot) {
   return (n.n_kv - 1) * nt_slot + own;
 }
 
-int choose_split(const sva_cache* c, long long units, int min_tiles) {
-  if (c->ws == nullptr) return 1;
+// Splits per work unit: the smallest s in 1..kMaxSplit minimising the wave
+// count per split, ceil(units * s / SMs) / s, subject to room for the split
+// items (`cap` of them; none without scratch) and to at least 4 key tiles
+// per split.
+int choose_split(const sva_cache* c, long long units, int min_tiles, long long cap) {
   const long long sms = c->num_sms;
   double best = (double)((units + sms - 1) / sms);
   int best_s = 1;
   for (int s = 2; s <= sva::kMaxSplit; ++s) {
     const long long items = units * s;
-    if (items > ws_items(c) || min_tiles / s < 4) break;
+    if (items > cap || min_tiles / s < 4) break;
     const double cost = (double)((items + sms - 1) / sms) / s;
     if (cost < best - 1e-9) {
       best = cost;
@@ -290,19 +301,20 @@ int choose_split(const sva_cache* c, long long units, int min_tiles) {
 }
 
 // The split plan of a launch: units 0..n_full-1 unsplit, the rest split
-// n_split ways.  When the units fill some whole waves of one CTA per SM, those
-// waves run unsplit and only the partial last wave is split; that has the
-// makespan of splitting every unit (when it is no longer) with fewer CTAs,
-// fewer prologues and epilogues and fewer partials to merge.
-void plan_split(const sva_cache* c, long long units, int min_tiles, long long* n_full,
-                int* n_split) {
+// n_split ways, with at most `cap` split items.  When the units fill some
+// whole waves of one CTA per SM, those waves run unsplit and only the partial
+// last wave is split; that has the makespan of splitting every unit (when it
+// is no longer) with fewer CTAs, fewer prologues and epilogues and fewer
+// partials to merge, and needs room for fewer split items.
+void plan_split(const sva_cache* c, long long units, int min_tiles, long long cap,
+                long long* n_full, int* n_split) {
   const long long sms = c->num_sms;
-  const int s_all = choose_split(c, units, min_tiles);
+  const int s_all = choose_split(c, units, min_tiles, cap);
   *n_full = 0;
   *n_split = s_all;
-  if (s_all == 1 || units < sms) return;
+  if (units < sms) return;
   const long long full = units / sms * sms, rest = units - full;
-  const int s_rest = choose_split(c, rest, min_tiles);
+  const int s_rest = choose_split(c, rest, min_tiles, cap);
   const double cost_all = (double)((units * s_all + sms - 1) / sms) / s_all;
   const double cost_mixed =
       (double)(full / sms) + (double)((rest * s_rest + sms - 1) / sms) / s_rest;
@@ -610,11 +622,18 @@ sva_status sva_rope_kv_write_qknorm(sva_cache* c, const sva_node* nodes, int32_t
 
 namespace {
 
-// sva_attend_nodes and sva_attend_nodes_sparse: the checks and the launch;
-// tile_mask and own_mask NULL is the dense mask.
+// Where the key-range split partials of an attention launch go.
+enum class Scratch {
+  kWorkspace,  // the caller's workspace (sva_cache_set_workspace), if attached
+  kStatic,     // the library's static device array (sva_attend_nodes_noalloc)
+};
+
+// sva_attend_nodes, _sparse, _masked and _noalloc: the checks, the launch
+// parameters, the split plan and the launch.  tile_mask and own_mask NULL is
+// the dense mask.  Every check runs before anything is enqueued.
 sva_status attend(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* q, void* out,
                   float* lse, float scale, const uint32_t* tile_mask, int32_t mask_words,
-                  const uint32_t* own_mask, int32_t own_words, sva_stream s) {
+                  const uint32_t* own_mask, int32_t own_words, sva_stream s, Scratch scratch) {
   if (c == nullptr || nodes == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "NULL argument");
   if (n_nodes < 1) return fail(SVA_ERR_INVALID_ARGUMENT, "n_nodes %d < 1", n_nodes);
   if (n_nodes > SVA_MAX_NODES)
@@ -702,6 +721,40 @@ sva_status attend(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const vo
       if ((long long)p.nodes[i].n_kv * p.nt_slot > 32LL * sva::kMaskWords)
         return fail(SVA_ERR_CAPACITY, "node %d: %lld key tiles exceed the %d a masked launch covers",
                     i, (long long)p.nodes[i].n_kv * p.nt_slot, 32 * sva::kMaskWords);
+
+  // The split plan.  The static scratch takes the plan a full caller
+  // workspace would get, so both entry points compute the same result, and
+  // refuses a plan whose partials do not fit the array.
+  int min_tiles = 1 << 30;
+  for (int i = 0; i < n_nodes; ++i)
+    min_tiles = std::min(min_tiles, key_tiles_walked(c, p.nodes[i], p.nt_slot));
+  p.n_qp = (p.n_qt + 1) / 2;
+  const long long units = (long long)g.num_heads * n_nodes * p.n_qp;
+  const long long cap = (scratch == Scratch::kStatic || c->ws != nullptr) ? ws_items(c) : 0;
+  long long n_full = 0;
+  int n_split = 1;
+  plan_split(c, units, min_tiles, cap, &n_full, &n_split);
+  char* split_base = c->ws;
+  size_t counter_bytes = ws_counter_bytes(c);
+  if (scratch == Scratch::kStatic) {
+    split_base = nullptr;
+    if (n_split > 1) {
+      const long long split_units = units - n_full;
+      counter_bytes = round_up((size_t)split_units * 4, 256);
+      const size_t need = counter_bytes + (size_t)split_units * n_split * ws_item_bytes(c);
+      if (need > sva::kStaticScratchBytes)
+        return fail(SVA_ERR_CAPACITY,
+                    "this launch splits %lld work units %d ways and needs %zu bytes of scratch; the "
+                    "library's static scratch holds %zu bytes (use sva_attend_nodes with a "
+                    "workspace for launches this large)",
+                    split_units, n_split, need, sva::kStaticScratchBytes);
+      void* addr = nullptr;
+      cudaError_t e = sva::static_split_scratch(c->device, &addr);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(split scratch)");
+      split_base = static_cast<char*>(addr);
+    }
+  }
+
   if (c->q_cached != q || c->q_cached_n != n_nodes) {
     st = encode_4d_q(&c->tmap_q, q, g, c->L.T, n_nodes);
     if (st != SVA_OK) {
@@ -720,27 +773,25 @@ sva_status attend(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const vo
   p.T = c->L.T;
   p.Tpad = c->L.Tpad;
   p.H = g.num_heads;
-  p.n_qp = (p.n_qt + 1) / 2;
   p.n_nodes = n_nodes;
   p.valid_last = c->L.T - (p.nt_slot - 1) * sva::kTile;
   p.frame_tokens = g.grid_h * g.grid_w;
-  p.fault_mode = c->fault_mode;
+  p.fault_mode = scratch == Scratch::kStatic ? 0 : c->fault_mode;
   p.timeout_ns = c->timeout_ns;
-  c->fault_mode = 0;
-  int min_tiles = 1 << 30;
-  for (int i = 0; i < n_nodes; ++i)
-    min_tiles = std::min(min_tiles, key_tiles_walked(c, p.nodes[i], p.nt_slot));
-  const long long units = (long long)g.num_heads * n_nodes * p.n_qp;
-  long long n_full = 0;
-  int n_split = 1;
-  plan_split(c, units, min_tiles, &n_full, &n_split);
+  if (scratch != Scratch::kStatic) c->fault_mode = 0;
   p.n_full = (int32_t)n_full;
   p.n_split = n_split;
-  if (p.n_split > 1) {
-    p.ws_count = reinterpret_cast<int*>(c->ws);
-    p.ws = reinterpret_cast<float*>(c->ws + ws_counter_bytes(c));
+  if (n_split > 1) {
+    p.ws_count = reinterpret_cast<int*>(split_base);
+    p.ws = reinterpret_cast<float*>(split_base + counter_bytes);
+    if (scratch == Scratch::kStatic) {
+      // the arrival counters must start at zero; the array keeps whatever the
+      // previous call left in it
+      cudaError_t e = cudaMemsetAsync(split_base, 0, counter_bytes, reinterpret_cast<cudaStream_t>(s));
+      if (e != cudaSuccess) return cuda_fail(e, "clearing the split counters");
+    }
   }
-  const long long grid = n_full + (units - n_full) * p.n_split;
+  const long long grid = n_full + (units - n_full) * n_split;
   cudaError_t e = sva::launch_attend(p, g.head_dim, (int)grid, reinterpret_cast<cudaStream_t>(s));
   if (e != cudaSuccess) return cuda_fail(e, "attend launch");
   return ok();
@@ -752,7 +803,8 @@ extern "C" {
 
 sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* q,
                             void* out, float* lse, float scale, sva_stream s) {
-  return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, s);
+  return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, s,
+                Scratch::kWorkspace);
 }
 
 }  // extern "C"
@@ -778,6 +830,16 @@ sva_status project(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const v
                      : "x, weight, q, k, v (and bias if given) must be non-NULL and 16-byte aligned");
   sva_status st = check_device(c);
   if (st != SVA_OK) return st;
+  {
+    // every operand must be memory of the cache's device: the tensor maps and
+    // the epilogue's stores address it directly
+    const void* ptrs[6] = {x, weight, bias, q, k, v};
+    const char* names[6] = {"x", "weight", "bias", rope ? "q_out" : "q", "k", "v"};
+    for (int i = 0; i < 6; ++i)
+      if (ptrs[i] != nullptr && !on_device(ptrs[i], c->device))
+        return fail(SVA_ERR_INVALID_ARGUMENT, "%s is not device memory of the cache's device %d",
+                    names[i], c->device);
+  }
   const sva_geometry& g = c->g;
   const int N = g.num_heads * g.head_dim;
   if (N % 128 != 0)
@@ -797,14 +859,15 @@ sva_status project(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const v
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return fail(SVA_ERR_CUDA, "cuTensorMapEncodeTiled(x) failed: %d", (int)r);
   }
-  {
+  for (int half = 0; half < 2; ++half) {
+    // W tiles of a whole item (BN rows) and of a half-width item (BN / 2)
     cuuint64_t dims[2] = {(cuuint64_t)in_features, (cuuint64_t)3 * N};
     cuuint64_t strides[1] = {(cuuint64_t)in_features * 2};
-    cuuint32_t box[2] = {64, (cuuint32_t)bn / 2};  // each CTA of a pair loads half a W tile
-    CUresult r = fn(&p.tmap_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(weight),
-                    dims, strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                    CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    cuuint32_t box[2] = {64, (cuuint32_t)(half ? bn / 2 : bn)};
+    CUresult r = fn(half ? &p.tmap_wh : &p.tmap_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                    const_cast<void*>(weight), dims, strides, box, es,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS)
       return fail(SVA_ERR_CUDA, "cuTensorMapEncodeTiled(weight) failed: %d", (int)r);
   }
@@ -854,9 +917,18 @@ sva_status project(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const v
   p.n_ntiles = 3 * N / bn;
   p.n_kblocks = (in_features + 63) / 64;
   p.timeout_ns = c->timeout_ns;
-  // clusters of two CTAs, each cluster one (pair of m tiles, n tile) at a time
-  const long long pairs = (long long)((p.n_mtiles + 1) / 2) * p.n_ntiles;
-  const int grid = 2 * (int)std::min<long long>(pairs, c->num_sms / 2);
+  // One CTA per SM walks the items.  The tiles of a partial last round are
+  // split into two half-width items when the halves fit one round (and, for
+  // the fused RoPE epilogue, still cover whole heads), so that the last round
+  // takes half as long.
+  const long long sms = c->num_sms;
+  const long long tiles = (long long)p.n_mtiles * p.n_ntiles;
+  if (tiles > INT32_MAX / 2) return fail(SVA_ERR_CAPACITY, "%lld output tiles", tiles);
+  const long long rest = tiles % sms;
+  const bool split_tail = rest > 0 && 2 * rest <= sms && (!rope || (bn / 2) % g.head_dim == 0);
+  p.n_whole = (int32_t)(split_tail ? tiles - rest : tiles);
+  p.n_items = (int32_t)(split_tail ? tiles + rest : tiles);
+  const int grid = (int)std::min<long long>(p.n_items, sms);
   cudaError_t e = sva::launch_qkv_project(p, bn, grid, reinterpret_cast<cudaStream_t>(s));
   if (e != cudaSuccess) return cuda_fail(e, "qkv_project launch");
   if (rope)
@@ -892,144 +964,29 @@ sva_status sva_attend_nodes_sparse(sva_cache* c, const sva_node* nodes, int32_t 
                                    const uint32_t* tile_mask, int32_t words_per_row,
                                    sva_stream s) {
   if (tile_mask == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "tile_mask is NULL");
-  return attend(c, nodes, n_nodes, q, out, lse, scale, tile_mask, words_per_row, nullptr, 0, s);
+  return attend(c, nodes, n_nodes, q, out, lse, scale, tile_mask, words_per_row, nullptr, 0, s,
+                Scratch::kWorkspace);
 }
 
 sva_status sva_attend_nodes_masked(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
                                    const void* q, void* out, float* lse, float scale,
                                    const sva_attn_mask* mask, sva_stream s) {
-  if (mask == nullptr) return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, s);
+  if (mask == nullptr)
+    return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, s,
+                  Scratch::kWorkspace);
   return attend(c, nodes, n_nodes, q, out, lse, scale, mask->tile_mask, mask->tile_words,
-                mask->own_mask, mask->own_words, s);
+                mask->own_mask, mask->own_words, s, Scratch::kWorkspace);
 }
 
 // Attention with the split scratch taken from the library's own device
-// array instead of a caller-attached workspace (see include/sva.h).  The
-// checks and the launch parameters are those of sva_attend_nodes.
+// array instead of a caller-attached workspace (see include/sva.h): the same
+// checks, the same split plan and the same kernel as sva_attend_nodes with a
+// workspace attached.
 sva_status sva_attend_nodes_noalloc(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
                                     const void* q, void* out, float* lse, float scale,
                                     sva_stream s) {
-  if (c == nullptr || nodes == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "NULL argument");
-  if (n_nodes < 1) return fail(SVA_ERR_INVALID_ARGUMENT, "n_nodes %d < 1", n_nodes);
-  if (n_nodes > SVA_MAX_NODES)
-    return fail(SVA_ERR_CAPACITY, "n_nodes %d > SVA_MAX_NODES (%d)", n_nodes, SVA_MAX_NODES);
-  if (q == nullptr || out == nullptr || !aligned16(q) || !aligned16(out) ||
-      (lse != nullptr && (reinterpret_cast<uintptr_t>(lse) & 3u) != 0))
-    return fail(SVA_ERR_INVALID_ARGUMENT, "q/out must be non-NULL and 16-byte aligned, lse 4-byte aligned");
-  if (!std::isfinite(scale) || !(scale > 0.0f))
-    return fail(SVA_ERR_INVALID_ARGUMENT, "scale must be finite and > 0");
-  sva_status st = check_device(c);
-  if (st != SVA_OK) return st;
-  const sva_geometry& g = c->g;
-
-  static thread_local sva::AttnParams p;
-  std::memset(&p, 0, sizeof(p));
-  for (int i = 0; i < n_nodes; ++i) {
-    const sva_node& n = nodes[i];
-    st = check_own(c, n, i, true);
-    if (st != SVA_OK) return st;
-    if (n.n_ctx < 0 || n.n_ctx > SVA_MAX_CTX)
-      return fail(SVA_ERR_CAPACITY, "node %d: n_ctx %d outside 0..%d", i, n.n_ctx, SVA_MAX_CTX);
-    if (n.within != SVA_WITHIN_BIDIRECTIONAL && n.within != SVA_WITHIN_FRAME_CAUSAL)
-      return fail(SVA_ERR_INVALID_ARGUMENT, "node %d: unknown within-chunk mode %d", i, n.within);
-    sva::AttnNode& a = p.nodes[i];
-    a.q_index = i;
-    a.frame_causal = n.within == SVA_WITHIN_FRAME_CAUSAL ? 1 : 0;
-    a.slot[0] = n.own_slot;
-    int nkv = 1;
-    for (int k = 0; k < n.n_ctx; ++k) {
-      const int32_t cs = n.ctx_slot[k];
-      if (cs < 0 || cs >= g.num_slots)
-        return fail(SVA_ERR_INVALID_ARGUMENT, "node %d ctx %d: slot %d out of range", i, k, cs);
-      const SlotInfo& si = c->slots[cs];
-      if (!si.bound || !si.resident)
-        return fail(SVA_ERR_NOT_RESIDENT, "node %d ctx %d: slot %d is %s", i, k, cs,
-                    si.bound ? "bound but not written" : "not bound");
-      if (si.seq != n.seq || si.chunk >= n.chunk)
-        return fail(SVA_ERR_CAUSALITY,
-                    "node %d (seq %d, chunk %d) ctx %d: slot %d holds (seq %d, chunk %d), not a "
-                    "past chunk of the same sequence",
-                    i, n.seq, n.chunk, k, cs, si.seq, si.chunk);
-      if (cs == n.own_slot)
-        return fail(SVA_ERR_INVALID_ARGUMENT, "node %d ctx %d repeats the own slot", i, k);
-      for (int k2 = 0; k2 < k; ++k2)
-        if (n.ctx_slot[k2] == cs)
-          return fail(SVA_ERR_INVALID_ARGUMENT, "node %d: slot %d listed twice", i, cs);
-      if (n.ctx_visible[k]) a.slot[nkv++] = cs;
-    }
-    a.n_kv = nkv;
-  }
-  p.n_qt = (c->L.T + sva::kTile - 1) / sva::kTile;
-  p.n_qp = (p.n_qt + 1) / 2;
-  p.nt_slot = c->L.Tpad / sva::kTile;
-  int min_tiles = 1 << 30;
-  for (int i = 0; i < n_nodes; ++i)
-    min_tiles = std::min(min_tiles, key_tiles_walked(c, p.nodes[i], p.nt_slot));
-  const long long units = (long long)g.num_heads * n_nodes * p.n_qp;
-
-  // The split plan a full workspace would get; its scratch must fit the array.
-  const long long sms = c->num_sms;
-  double best = (double)((units + sms - 1) / sms);
-  int n_split = 1;
-  for (int sp = 2; sp <= sva::kMaxSplit; ++sp) {
-    const long long items = units * sp;
-    if (items > ws_items(c) || min_tiles / sp < 4) break;
-    const double cost = (double)((items + sms - 1) / sms) / sp;
-    if (cost < best - 1e-9) {
-      best = cost;
-      n_split = sp;
-    }
-  }
-  void* scratch = nullptr;
-  size_t counter_bytes = 0;
-  if (n_split > 1) {
-    counter_bytes = round_up((size_t)units * 4, 256);
-    const size_t need = counter_bytes + (size_t)units * n_split * ws_item_bytes(c);
-    if (need > sva::kStaticScratchBytes)
-      return fail(SVA_ERR_CAPACITY,
-                  "this launch splits %lld work units %d ways and needs %zu bytes of scratch; the "
-                  "library's static scratch holds %zu bytes (use sva_attend_nodes with a "
-                  "workspace for launches this large)",
-                  units, n_split, need, sva::kStaticScratchBytes);
-    cudaError_t e = sva::static_split_scratch(c->device, &scratch);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(split scratch)");
-    // the arrival counters must start at zero; the array keeps whatever the
-    // previous call left in it
-    e = cudaMemsetAsync(scratch, 0, counter_bytes, reinterpret_cast<cudaStream_t>(s));
-    if (e != cudaSuccess) return cuda_fail(e, "clearing the split counters");
-  }
-  if (c->q_cached != q || c->q_cached_n != n_nodes) {
-    st = encode_4d_q(&c->tmap_q, q, g, c->L.T, n_nodes);
-    if (st != SVA_OK) {
-      c->q_cached = nullptr;
-      return st;
-    }
-    c->q_cached = q;
-    c->q_cached_n = n_nodes;
-  }
-  p.tmap_q = c->tmap_q;
-  p.tmap_kv = c->tmap_kv;
-  p.out = out;
-  p.lse = lse;
-  p.status = reinterpret_cast<int*>(c->base + c->L.status);
-  p.scale_log2 = scale * 1.4426950408889634f;
-  p.T = c->L.T;
-  p.Tpad = c->L.Tpad;
-  p.H = g.num_heads;
-  p.n_nodes = n_nodes;
-  p.valid_last = c->L.T - (p.nt_slot - 1) * sva::kTile;
-  p.frame_tokens = g.grid_h * g.grid_w;
-  p.fault_mode = 0;
-  p.timeout_ns = c->timeout_ns;
-  p.n_split = n_split;
-  if (n_split > 1) {
-    p.ws_count = static_cast<int*>(scratch);
-    p.ws = reinterpret_cast<float*>(static_cast<char*>(scratch) + counter_bytes);
-  }
-  const long long grid = units * n_split;
-  cudaError_t e = sva::launch_attend(p, g.head_dim, (int)grid, reinterpret_cast<cudaStream_t>(s));
-  if (e != cudaSuccess) return cuda_fail(e, "attend launch");
-  return ok();
+  return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, s,
+                Scratch::kStatic);
 }
 
 sva_status sva_poll_device_status(sva_cache* c, sva_stream s) {
