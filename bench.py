@@ -35,10 +35,13 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "chunk-attention TFLOP/s (% of GB300 BF16 peak) and denoising nodes/s per layer"
-DEFAULT_WORKLOAD = "clean1"
+DEFAULT_WORKLOAD = "stress14b"
 KERNEL_SOURCES = ["paper_2609_22283_gb300/csrc/attend.cu", "paper_2609_22283_gb300/csrc/ptx.cuh",
                   "paper_2609_22283_gb300/csrc/internal.h"]
-TRAFFIC_FILE = os.path.join(ROOT, "profiles", "attend_dram_traffic.md")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "attend_dram_traffic.json")
+# Further full-geometry configurations timed beside the default one (attention
+# and RoPE + cache write only), each in the same run.
+PER_CONFIG = ("clean1", "same4", "prog4")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -112,19 +115,20 @@ def kernel_hash() -> str:
 
 
 def read_traffic(workload: str):
-    """DRAM bytes per attend launch from the committed ncu summary, if it was
-    taken on the current kernel source (matching hash); else None."""
+    """DRAM bytes per attend launch from the committed ncu table
+    (profiles/attend_dram_traffic.json), if it was taken on the current
+    kernel code (matching hash); else None."""
     try:
-        text = open(TRAFFIC_FILE).read()
-    except OSError:
+        with open(TRAFFIC_FILE) as f:
+            table = json.load(f)
+    except (OSError, ValueError):
         return None
     want = kernel_hash()
-    for line in text.splitlines():
-        parts = [p.strip() for p in line.strip().strip("|").split("|")]
-        if len(parts) >= 3 and parts[0] == workload and parts[1] == want:
+    for row in table.get("rows", []):
+        if row.get("workload") == workload and row.get("kernel_hash") == want:
             try:
-                return float(parts[2])
-            except ValueError:
+                return float(row["dram_bytes_per_launch"])
+            except (KeyError, TypeError, ValueError):
                 return None
     return None
 
@@ -240,11 +244,14 @@ def oracle_sample(w, inp, seconds: float, min_rows: int = 16):
 
     oracle.build()
     g = oracle.Geometry(F=w.F, Hp=w.Hp, Wp=w.Wp, H=w.H, d=w.d, pairs=w.pairs, theta=w.theta)
-    states = {k: (a.to(torch.float64).numpy(), b.to(torch.float64).numpy())
-              for k, (a, b) in I.all_states(w, inp).items()}
+    # node 0's sequence only, as fp32 (bf16 values exactly; the oracle widens
+    # each head it reads to fp64)
+    seq0 = w.nodes[0][0]
+    states = {k: (a.float().numpy(), b.float().numpy())
+              for k, (a, b) in I.all_states(w, inp).items() if k[0] == seq0}
     (_, b, _) = w.nodes[0]
     lkv = w.T * (1 + max(0, min(w.W, b - 1)))
-    q = inp.q[0].to(torch.float64).numpy()
+    q = inp.q[0].float().numpy()
     rng = np.random.default_rng(5)
     rows_done, spent = 0, 0.0
     batch = min_rows
@@ -308,6 +315,17 @@ def config_of(w, world):
 
 
 # ---------------------------------------------------------------- GPU arm
+
+def plan_extras(args, world: int, rank: int, workload: str) -> dict:
+    """Which measurements run beside the timed step.  The QKV projection and
+    the other configurations are timed on a single GPU only (under torchrun
+    each rank runs an independent replica of the step and nothing else); the
+    oracle's CPU baseline runs on rank 0 of a single-GPU run."""
+    single = world == 1
+    return {"projection": single and not args.no_projection,
+            "per_config": single and not args.no_per_config and workload not in PER_CONFIG,
+            "cpu_baseline": single and rank == 0 and not args.no_cpu_baseline}
+
 
 def run_ours(args, world, rank, local):
     import torch
@@ -499,7 +517,10 @@ def run_ours(args, world, rank, local):
     }
     if remeasured:
         line["clocks_note"] = "first timed region saw a slowdown reason; re-measured once"
-    if not args.no_projection:
+    extras = plan_extras(args, world, rank, w.name)
+    if extras["per_config"]:
+        line["per_config"] = {}
+    if extras["projection"]:
         line["qkv_project"] = time_projection(step, w, dev, flush, stream, peak, world)
         # the attention layer's three device steps: projection, RoPE + cache
         # write, attention (kernel times summed; the projection is not in `value`)
@@ -511,7 +532,13 @@ def run_ours(args, world, rank, local):
                                                    fused=True)
         line["nodes_per_s_fused_layer"] = (
             w.n_nodes * world / ((line["qkv_project_rope"]["ms"] + t_attn_ms) * 1e-3))
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if "per_config" in line:
+        step.close()
+        step = None
+        for name in PER_CONFIG:
+            line["per_config"][name] = time_config(I.WORKLOADS[name], dev, flush, stream, peak,
+                                                   min(args.steps, 20), args.warmup)
+    if extras["cpu_baseline"]:
         tf, rows, secs, cores = oracle_sample(w, inp, args.cpu_seconds)
         line["cpu_baseline"] = {
             "value": tf, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
@@ -519,8 +546,49 @@ def run_ours(args, world, rank, local):
                       f"(fp64 C oracle, OpenMP; incl. its RoPE of the node's key states)"}
     if rank == 0:
         print(json.dumps(line), flush=True)
-    step.close()
+    if step is not None:
+        step.close()
     return 0
+
+
+def time_config(w, dev, flush, stream, peak, K, warmup):
+    """Attention and RoPE + cache write of another workload, timed like the
+    main step (CUDA events per kernel, L2 flushed between steps)."""
+    import torch
+    from paper_2609_22283_gb300 import inputs as I
+    from paper_2609_22283_gb300.pipeline import Step
+    inp = I.generate(w)
+    step = Step(w, device=str(dev))
+    step.prefill(inp)
+    q, k, v = step.device_inputs(inp)
+    out, lse = step.outputs()
+    for _ in range(warmup):
+        nodes_, _ = step.node_table()
+        step.cache.rope_kv_write(nodes_, k, v, q, check=False)
+        step.attend(nodes_, q, out, lse)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    torch.cuda.synchronize()
+    for i in range(K):
+        flush()
+        nodes_, _ = step.node_table()
+        ev[i][0].record(stream)
+        step.cache.rope_kv_write(nodes_, k, v, q, check=False)
+        ev[i][1].record(stream)
+        step.attend(nodes_, q, out, lse)
+        ev[i][2].record(stream)
+    torch.cuda.synchronize()
+    if step.cache.poll() != 0:
+        raise RuntimeError(f"device status after timing {w.name}")
+    rope_ms = sum(e[0].elapsed_time(e[1]) for e in ev) / K
+    attn_ms = sum(e[1].elapsed_time(e[2]) for e in ev) / K
+    step.close()
+    flops = attn_flops(w)
+    tf = flops / (attn_ms * 1e-3) / 1e12
+    return {"attend_ms": attn_ms, "achieved": tf, "unit": "TFLOP/s", "frac": tf / peak,
+            "rope_ms": rope_ms, "rope_gbs": rope_bytes(w) / (rope_ms * 1e-3) / 1e9,
+            "nodes_per_s": w.n_nodes / ((rope_ms + attn_ms) * 1e-3), "steps": K,
+            "kv_tokens_per_node": [w.T * (1 + max(0, min(w.W, b - 1))) for (_, b, _) in w.nodes],
+            "nodes": w.n_nodes, "heads": w.H}
 
 
 def time_projection(step, w, dev, flush, stream, peak, world, fused=False):
@@ -529,7 +597,10 @@ def time_projection(step, w, dev, flush, stream, peak, world, fused=False):
     step: CUDA events per launch, L2 flushed between launches.  Reported
     beside the step, not inside it.  With `fused`, sva_qkv_project_rope: the
     same projection with the RoPE + cache write in its epilogue (it writes the
-    nodes' own slots; run after every timed step and check)."""
+    nodes' own slots; run after every timed step and check).  Single GPU
+    only: replica runs under torchrun never call it."""
+    if world != 1:
+        raise RuntimeError("the projection is timed on a single GPU only")
     import torch
     from paper_2609_22283_gb300 import inputs as I
     C = w.H * w.d
@@ -570,7 +641,9 @@ def compare_schedules(args):
     """Per-chunk attention-layer time of the two executions of Table 3 (Section 5),
     on one GPU: fully serial clean history (Eq. 5; five one-node launches per
     chunk: four denoising updates and the clean refresh, W = 6) against the
-    progressive pipeline (one launch of a round's four nodes plus the refresh)."""
+    progressive pipeline (one launch of a round's four nodes plus the refresh).
+    Each chunk is timed as a whole (CUDA events around it, L2 flushed before
+    it) and each launch in it on its own (events around every launch)."""
     import torch
 
     import __graft_entry__
@@ -581,7 +654,7 @@ def compare_schedules(args):
     torch.cuda.set_device(0)
     stream = torch.cuda.current_stream()
     flush = L2Flush("cuda")
-    res = {}
+    res, launches, clocks = {}, {}, {}
     for name in ("clean5", "prog4r"):
         w = I.WORKLOADS[name]
         inp = I.generate(w)
@@ -591,33 +664,47 @@ def compare_schedules(args):
         out, lse = step.outputs()
         nodes, n = step.node_table()
 
-        def one_chunk():
+        def one_chunk(evs=None):
+            def rec():
+                if evs is not None:
+                    e = torch.cuda.Event(enable_timing=True)
+                    e.record(stream)
+                    evs.append(e)
+            rec()
             if name == "clean5":                        # one launch per node, in order
                 for i in range(n):
                     sl = slice(i, i + 1)
-                    one = nodes[i:i + 1]
-                    arr = (type(nodes[0]) * 1)(one[0])
-                    step.cache.rope_kv_write(arr, k[sl], v[sl], q[sl], check=False)
-                    step.cache.attend_nodes(arr, q[sl], out[sl], lse[sl], step.scale, check=False)
+                    one = (type(nodes[0]) * 1)(nodes[i])
+                    step.cache.rope_kv_write(one, k[sl], v[sl], q[sl], check=False)
+                    rec()
+                    step.cache.attend_nodes(one, q[sl], out[sl], lse[sl], step.scale, check=False)
+                    rec()
             else:
                 step.cache.rope_kv_write(nodes, k, v, q, check=False)
+                rec()
                 step.cache.attend_nodes(nodes, q, out, lse, step.scale, check=False)
+                rec()
 
         for _ in range(args.warmup):
             one_chunk()
-        total = 0.0
+        sampler = ClockSampler(0)
+        sampler.start()
+        time.sleep(0.3)
+        total, per = 0.0, None
         for _ in range(args.steps):
             flush()
-            e0 = torch.cuda.Event(enable_timing=True)
-            e1 = torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            one_chunk()
-            e1.record(stream)
+            evs = []
+            one_chunk(evs)
             torch.cuda.synchronize()
-            total += e0.elapsed_time(e1)
+            total += evs[0].elapsed_time(evs[-1])
+            t = [a.elapsed_time(b) for a, b in zip(evs[:-1], evs[1:])]
+            per = t if per is None else [x + y for x, y in zip(per, t)]
+        clocks[name] = sampler.stop()
         if step.cache.poll() != 0:
             raise RuntimeError("device status after timing")
         res[name] = total / args.steps
+        kinds = ["rope_kv_write", "attend_nodes"] * (n if name == "clean5" else 1)
+        launches[name] = [{"kernel": kd, "ms": x / args.steps} for kd, x in zip(kinds, per)]
         step.close()
     line = {"metric": "attention-layer time per chunk (RoPE + cache write + attention), ms",
             "clean_serial_ms": res["clean5"], "progressive_pipeline_ms": res["prog4r"],
@@ -625,13 +712,15 @@ def compare_schedules(args):
             "steps": args.steps, "warmup": args.warmup, "n_gpus": 1, "data": "synthetic",
             "config": {"serial": I.WORKLOADS["clean5"].description,
                        "pipeline": I.WORKLOADS["prog4r"].description},
+            "launches": launches, "clocks": clocks,
+            "l2": "flushed before each timed chunk (256 MiB write, then a 256 MiB read)",
             "paper_context": "full-DiT steady-state speedup 1.57-2.83x on 4-12 Ascend 910B2C with "
                              "context parallelism (Table 3); not the same measurement"}
     print(json.dumps(line), flush=True)
     return 0
 
 
-def main():
+def parse_args(argv=None):
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=2000)
@@ -643,11 +732,18 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-projection", action="store_true",
                     help="skip timing the QKV projection beside the step")
+    ap.add_argument("--no-per-config", action="store_true",
+                    help="skip timing the other full-geometry configurations beside the step")
     ap.add_argument("--compare-schedules", action="store_true",
                     help="time clean-serial against progressive-pipeline execution of one chunk")
-    args = ap.parse_args()
+    args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
+    return args
+
+
+def main():
+    args = parse_args()
     if args.compare_schedules:
         return compare_schedules(args)
     world, rank, local = dist_setup()

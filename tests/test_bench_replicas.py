@@ -25,6 +25,16 @@ def _worker(rank, world, port, out):
     assert (w, r, l) == (world, rank, rank)
     bench.barrier(w)
     t = bench.reduce_max(1.5 + rank, w)       # per-rank step times 1.5 and 2.5 ms
+    # a replica run measures the step only: no projection (nor the other
+    # configurations or the CPU baseline), whatever the flags say
+    extras = bench.plan_extras(bench.parse_args([]), w, r, "stress14b")
+    assert extras == {"projection": False, "per_config": False, "cpu_baseline": False}, extras
+    try:
+        bench.time_projection(None, None, None, None, None, 0.0, w)
+        reached = True
+    except RuntimeError:
+        reached = False
+    assert not reached
     out[rank] = t
     import torch.distributed as dist
     dist.destroy_process_group()
@@ -41,6 +51,16 @@ def test_two_replicas_take_the_max_step_time():
         p.join(timeout=120)
         assert p.exitcode == 0
     assert out[0] == pytest.approx(2.5) and out[1] == pytest.approx(2.5)
+
+
+def test_single_gpu_runs_the_extras():
+    import bench
+    args = bench.parse_args([])
+    assert bench.plan_extras(args, 1, 0, "stress14b") == {
+        "projection": True, "per_config": True, "cpu_baseline": True}
+    args = bench.parse_args(["--no-projection", "--no-per-config", "--no-cpu-baseline"])
+    assert not any(bench.plan_extras(args, 1, 0, "stress14b").values())
+    assert bench.DEFAULT_WORKLOAD == "stress14b"
 
 
 def test_config_describes_replicas():
