@@ -122,6 +122,6 @@ cudaError_t static_split_scratch(int device, void** ptr);
 
 // Launchers (defined in the .cu files).  They return the launch error.
 cudaError_t launch_attend(const AttnParams& p, int head_dim, int grid, cudaStream_t s);
-cudaError_t launch_rope_kv(const RopeParams& p, cudaStream_t s);
+cudaError_t launch_rope_kv(const RopeParams& p, int num_sms, cudaStream_t s);
 
 }  // namespace sva

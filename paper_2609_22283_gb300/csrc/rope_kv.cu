@@ -67,7 +67,14 @@ __device__ __forceinline__ uint32_t rotate_pair(uint32_t xy, float c, float s) {
 // token-major inputs, so the warp walks them as 16-byte vectors; lane l always
 // holds vector l mod (d/8) of a head row, i.e. the same four pairs for every
 // head, so its cos/sin come from the tables once per token.
-__global__ void __launch_bounds__(256) rope_kv_kernel(const __grid_constant__ RopeParams p) {
+// Instances: with the RMSNorm of K (and Q), and two without it.  kWave
+// holds the kernel to 64 registers (loads in batches of two), so four
+// 256-thread blocks fit an SM and a launch of one 4680-token node (585
+// blocks) runs in a single wave: such a launch is bound by memory latency,
+// and occupancy is what hides it.  Larger launches loop over their tokens
+// and do better with batches of four at two blocks per SM.
+template <bool kNorm, bool kWave>
+__global__ void __launch_bounds__(256, kWave ? 4 : 2) rope_kv_kernel(const __grid_constant__ RopeParams p) {
   const int lane = threadIdx.x & 31;
   const int vpr = p.d >> 3;                        // 16-byte vectors per (token, head) row
   const int vshift = (vpr == 16) ? 4 : 3;
@@ -108,8 +115,8 @@ __global__ void __launch_bounds__(256) rope_kv_kernel(const __grid_constant__ Ro
     // RMSNorm scale of the token's K and Q vectors (pass over the row, then a
     // warp reduction); the second pass below reloads the row from L1/L2.
     float rk = 1.0f, rq = 1.0f;
-    const bool norm = p.gamma_k != nullptr;
-    if (norm) {
+    constexpr bool norm = kNorm;
+    if constexpr (norm) {
       float sk = 0.0f, sq = 0.0f;
       for (int v = lane; v < per_tok; v += 32) {
         const size_t off = in_tok + (size_t)v * 8;
@@ -128,7 +135,9 @@ __global__ void __launch_bounds__(256) rope_kv_kernel(const __grid_constant__ Ro
     // Batches of kBatch vectors per lane: every load of a batch is issued
     // before any of its stores (q is rotated in place, so without the split
     // the compiler keeps each iteration's loads behind the previous stores).
-    constexpr int kBatch = 4;
+    // The single-wave instance runs four blocks per SM, so half the batch
+    // keeps as many bytes in flight per SM as the others' two blocks.
+    constexpr int kBatch = kWave ? 2 : 4;
     for (int v0 = lane; v0 < per_tok; v0 += 32 * kBatch) {
       uint4 kv[kBatch], vv[kBatch], qv[kBatch];
 #pragma unroll
@@ -149,7 +158,7 @@ __global__ void __launch_bounds__(256) rope_kv_kernel(const __grid_constant__ Ro
         const size_t in_off = in_tok + (size_t)v * 8;
         uint32_t kw[4] = {kv[j].x, kv[j].y, kv[j].z, kv[j].w};
         uint32_t qw[4] = {qv[j].x, qv[j].y, qv[j].z, qv[j].w};
-        if (norm) {
+        if constexpr (norm) {
           const float4* gk = reinterpret_cast<const float4*>(p.gamma_k + (size_t)v * 8);
           const float4 gk0 = __ldg(gk), gk1 = __ldg(gk + 1);
           const float gkk[8] = {gk0.x, gk0.y, gk0.z, gk0.w, gk1.x, gk1.y, gk1.z, gk1.w};
@@ -183,8 +192,14 @@ __global__ void __launch_bounds__(256) rope_kv_kernel(const __grid_constant__ Ro
 
 }  // namespace
 
-cudaError_t launch_rope_kv(const RopeParams& p, cudaStream_t s) {
-  rope_kv_kernel<<<p.grid_blocks, 256, 0, s>>>(p);
+cudaError_t launch_rope_kv(const RopeParams& p, int num_sms, cudaStream_t s) {
+  const long long blocks = ((long long)p.n_nodes * p.T + 7) / 8;  // one warp per token
+  if (p.gamma_k != nullptr)
+    rope_kv_kernel<true, false><<<p.grid_blocks, 256, 0, s>>>(p);
+  else if (blocks <= 4LL * num_sms)
+    rope_kv_kernel<false, true><<<p.grid_blocks, 256, 0, s>>>(p);
+  else
+    rope_kv_kernel<false, false><<<p.grid_blocks, 256, 0, s>>>(p);
   return cudaGetLastError();
 }
 

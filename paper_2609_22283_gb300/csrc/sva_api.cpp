@@ -590,7 +590,7 @@ sva_status rope_write(sva_cache* c, const sva_node* nodes, int32_t n_nodes, cons
   const long long tokens = (long long)n_nodes * p.T;  // one warp per token, 8 warps per block
   const long long blocks = (tokens + 7) / 8;
   p.grid_blocks = (int)std::min<long long>(blocks, (long long)c->num_sms * 16);
-  cudaError_t e = sva::launch_rope_kv(p, reinterpret_cast<cudaStream_t>(s));
+  cudaError_t e = sva::launch_rope_kv(p, c->num_sms, reinterpret_cast<cudaStream_t>(s));
   if (e != cudaSuccess) return cuda_fail(e, "rope_kv launch");
   for (int i = 0; i < n_nodes; ++i) c->slots[nodes[i].own_slot].resident = true;
   return ok();

@@ -51,7 +51,9 @@ def _check_rotated(got, ref, raw, what):
     assert exact >= 0.999, f"{what}: only {exact:.5f} exact"
 
 
-@pytest.mark.parametrize("name", ["tiny", "clean1"])
+# tiny and clean1 take the single-wave instance of the RoPE kernel, prog4
+# (18720 tokens) the one for larger launches
+@pytest.mark.parametrize("name", ["tiny", "clean1", "prog4"])
 def test_cache_indexing_and_rope(oracle_mod, name):
     w = I.WORKLOADS[name]
     inp = I.generate(w)
