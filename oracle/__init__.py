@@ -244,7 +244,7 @@ def attend_rows(q: np.ndarray, k: np.ndarray, v: np.ndarray, scale: float,
 def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
                  states: dict, q_raw: np.ndarray, heads, rows, scale: float,
                  hidden: frozenset = frozenset(), within: str = "bidirectional",
-                 norm=None, tile_mask=None, own_mask=None):
+                 norm=None, tile_mask=None, own_mask=None, hist_mask=None):
     """One denoising node (seq, b, j), computed from raw (pre-RoPE) inputs.
 
     states: {(seq, chunk, level): (K_raw, V_raw)} with arrays [T][H][d] holding
@@ -266,6 +266,10 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
     own_mask: None, or a boolean array [T][T] for the node: query u sees key v
         of its own chunk only if own_mask[u][v] (the general token-level M of
         Eq. 4 inside the chunk); a further mask on top of the others.
+    hist_mask: None, or a boolean array [n_sel][T][T] for the node: query u
+        sees key token v of the j-th selected state (Eq. 2's offset order, j = 0
+        for r = 1) only if hist_mask[j][u][v] (the token-level M of Eq. 4 on
+        the history); a further mask on top of the others.
 
     Steps (Section 3.2): select the context states of the node with Eq. 2-3;
     rotate the K of the node's own state and of every selected state and the
@@ -294,7 +298,7 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
     row_frame = rows // frame_tokens if within == "frame_causal" else np.zeros_like(rows)
     row_tile = rows // 128 if tile_mask is not None else np.zeros_like(rows)
     groups = []
-    if own_mask is not None:       # every row its own mask
+    if own_mask is not None or hist_mask is not None:   # every row its own mask
         for r in range(len(rows)):
             groups.append((row_frame[r] if within == "frame_causal" else None,
                            row_tile[r] if tile_mask is not None else None, np.array([r])))
@@ -332,6 +336,11 @@ def node_forward(g: Geometry, policy: int, W: int, node: tuple[int, int, int],
             if own_mask is not None:
                 u = rows[idx[0]]
                 m[:g.T] = np.where(np.asarray(own_mask[u], dtype=bool), m[:g.T], -np.inf)
+            if hist_mask is not None:
+                u = rows[idx[0]]
+                for si in range(1, len(key_states)):     # selected state si - 1
+                    seg = slice(si * g.T, (si + 1) * g.T)
+                    m[seg] = np.where(np.asarray(hist_mask[si - 1][u], dtype=bool), m[seg], -np.inf)
             o, l = attend_rows(q[idx], k, v, scale, m)
             out[hi, idx] = o
             lse[hi, idx] = l

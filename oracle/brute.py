@@ -72,7 +72,7 @@ def _rope(x: np.ndarray, chunk: int, F: int, Hp: int, Wp: int, pairs, theta: flo
 def brute_forward(policy: str, W: int, F: int, Hp: int, Wp: int, pairs, theta: float,
                   node: tuple[int, int, int], grid: dict, q_raw: np.ndarray,
                   heads, scale: float, hidden=frozenset(), frame_causal: bool = False,
-                  tile_mask=None, own_mask=None):
+                  tile_mask=None, own_mask=None, hist_mask=None):
     """All query rows of `heads` for node (seq, b, j) against the whole grid.
 
     grid: {(seq, chunk, level): (K_raw, V_raw)} [T][H][d]; it may hold states
@@ -85,6 +85,9 @@ def brute_forward(policy: str, W: int, F: int, Hp: int, Wp: int, pairs, theta: f
     set, r = b - c (the offset of Eq. 2; 0 for the own chunk), nt = ceil(T/128).
     own_mask: None, or booleans [T][T]: query u sees key token v of its own
     chunk only if own_mask[u][v].
+    hist_mask: None, or booleans [n][T][T]: query u sees key token v of state
+    (c, l) with r = b - c >= 1 only if hist_mask[r - 1][u][v] (past the
+    window the state is masked anyway).
     Returns (out [len(heads)][T][d], lse [len(heads)][T]).
     """
     seq, b, j = node
@@ -120,6 +123,14 @@ def brute_forward(policy: str, W: int, F: int, Hp: int, Wp: int, pairs, theta: f
                 for v in range(T):
                     if not own_mask[u][v]:
                         Mu[own_start + v] = -np.inf
+            if hist_mask is not None:
+                for ki, (s, c, l) in enumerate(keys):
+                    r = b - c
+                    if s != seq or r < 1 or r > len(hist_mask):
+                        continue   # the own chunk, other sequences, future and far chunks
+                    for v in range(T):
+                        if not hist_mask[r - 1][u][v]:
+                            Mu[ki * T + v] = -np.inf
             if tile_mask is not None:
                 for ki, (s, c, l) in enumerate(keys):
                     if s != seq or not (0 <= b - c) or (b - c) * nt >= len(tile_mask[0]):

@@ -330,3 +330,73 @@ def test_own_token_mask_special_cases(oracle_mod):
     z, lz, _ = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), [130], 0.125,
                                        own_mask=none)
     assert not np.allclose(z, base[:, 2:3])
+
+
+def _hist_mask(n, T, seed, density=0.5):
+    rng = np.random.default_rng(seed)
+    m = rng.random((n, T, T)) < density
+    m[:, 7, :] = False                         # row 7 sees no history key
+    return m
+
+
+@pytest.mark.parametrize("within", ["bidirectional", "frame_causal"])
+def test_history_token_mask_against_dense_brute_force(oracle_mod, within):
+    """The token-level M of Eq. 4 on the history: the oracle's slot-list form
+    against the dense mask over the whole (chunk, level) grid, alone and with
+    an own-chunk token mask and a block-sparse tile mask."""
+    from oracle import brute
+    w, inp, g, states, masks = _sparse_case(oracle_mod, within)
+    rng = np.random.default_rng(8)
+    grid = dict(states)
+    for s in [(0, 2, 0), (0, 4, 0)]:
+        grid[s] = (rng.standard_normal((w.T, w.H, w.d)), rng.standard_normal((w.T, w.H, w.d)))
+    scale = 1.0 / math.sqrt(w.d)
+    rows = [0, 1, 5, 7, 64, 127, 128, 200, 255, 256, 300, w.T - 1]
+    for i, node in enumerate(w.nodes):
+        n_sel = max(0, min(w.W, node[1] - 1))
+        hist = _hist_mask(max(n_sel, 1), w.T, 20 + i)
+        own = _own_mask(w.T, 30 + i)
+        q = _f64(inp.q[i])
+        for own_m, tm in ((None, None), (own, masks[i])):
+            out, lse, _ = oracle_mod.node_forward(g, oracle_mod.POLICY_IDS[w.policy], w.W, node, states,
+                                                  q, range(w.H), rows, scale, within=within,
+                                                  tile_mask=tm, own_mask=own_m, hist_mask=hist)
+            bo, bl = brute.brute_forward(w.policy, w.W, w.F, w.Hp, w.Wp, w.pairs, w.theta, node, grid,
+                                         q, range(w.H), scale, frame_causal=within == "frame_causal",
+                                         tile_mask=tm, own_mask=own_m, hist_mask=hist)
+            np.testing.assert_allclose(out, bo[:, rows], rtol=0, atol=1e-12)
+            np.testing.assert_allclose(lse, bl[:, rows], rtol=0, atol=1e-12)
+
+
+def test_history_token_mask_special_cases(oracle_mod):
+    """An all-true history mask is the unmasked node; a state whose bits are
+    all clear for every row is that state hidden (ctx_visible = 0); a row
+    with no history bit sees its own chunk alone."""
+    w, inp, g, states, _ = _sparse_case(oracle_mod, "bidirectional")
+    pol = oracle_mod.POLICY_IDS[w.policy]
+    node = w.nodes[0]
+    q = _f64(inp.q[0])
+    rows = [0, 5, 130, w.T - 1]
+    n_sel = max(0, min(w.W, node[1] - 1))
+    assert n_sel == 2
+    base, bl, sel = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), rows, 0.125)
+    ones = np.ones((n_sel, w.T, w.T), bool)
+    a, la, _ = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), rows, 0.125,
+                                       hist_mask=ones)
+    np.testing.assert_array_equal(a, base)
+    np.testing.assert_array_equal(la, bl)
+    second_off = ones.copy()
+    second_off[1] = False
+    b, lb2, _ = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), rows, 0.125,
+                                        hist_mask=second_off)
+    hid, lh, _ = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), rows, 0.125,
+                                         hidden=frozenset({sel[1]}))
+    np.testing.assert_array_equal(b, hid)
+    np.testing.assert_array_equal(lb2, lh)
+    no_hist = np.zeros((n_sel, w.T, w.T), bool)
+    c, lc, _ = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), rows, 0.125,
+                                       hist_mask=no_hist)
+    own_alone, lo, _ = oracle_mod.node_forward(g, pol, w.W, node, states, q, range(w.H), rows, 0.125,
+                                               hidden=frozenset(sel))
+    np.testing.assert_array_equal(c, own_alone)
+    assert not np.allclose(c, base)
