@@ -298,19 +298,28 @@ typedef struct {
    * token v of its own chunk.  own_words >= ceil(T / 32); 4-byte aligned. */
   const uint32_t* own_mask;
   int32_t own_words;
+  /* Token-level visibility of the history: device array of 32-bit words
+   * [n_nodes][T][hist_states][hist_words]; bit v of row (node i, query token
+   * u, context j) set means query u of node i may attend key token v of the
+   * state in nodes[i].ctx_slot[j].  hist_states >= n_ctx of every node (and
+   * >= 1), hist_words >= ceil(T / 32); 4-byte aligned. */
+  const uint32_t* hist_mask;
+  int32_t hist_states;
+  int32_t hist_words;
 } sva_attn_mask;
 
 /* sva_attend_nodes with the general token-level mask M of Eq. 4 (Section
- * 3.2) inside the own chunk and/or query-dependent block-sparse access to
- * the history: M(u, v) = -inf where the own-chunk bit of (u, v) or the tile
- * bit of (u's query tile, v's key tile) is clear, on top of every other mask
- * (hidden context slots, the within-chunk mode, padding).  The frame-causal
+ * 3.2) inside the own chunk and on the history, and/or query-dependent
+ * block-sparse access to the history: M(u, v) = -inf where the own-chunk or
+ * history bit of (u, v) or the tile bit of (u's query tile, v's key tile) is
+ * clear, on top of every other mask (hidden context slots, the within-chunk
+ * mode, padding).  The frame-causal
  * mode is the own mask with bit v set iff v's latent frame is not after u's.
  * Queries that see no key get O = 0 and LSE = -inf.  Both masks are read by
  * the kernel on `s` and must stay valid until it completes.  Errors: as
- * sva_attend_nodes_sparse, plus INVALID_ARGUMENT for a misaligned own mask
- * or a short own row; a NULL mask pointer or two NULL masks is plain
- * sva_attend_nodes. */
+ * sva_attend_nodes_sparse, plus INVALID_ARGUMENT for a misaligned token mask,
+ * a short row or too few history states; a NULL mask pointer or three NULL
+ * masks is plain sva_attend_nodes. */
 sva_status sva_attend_nodes_masked(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
                                    const void* q, void* out, float* lse, float scale,
                                    const sva_attn_mask* mask, sva_stream s);

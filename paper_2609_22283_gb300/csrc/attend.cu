@@ -559,17 +559,24 @@ __global__ void __launch_bounds__(kThreads, 1) attend_kernel(const __grid_consta
 #pragma unroll
       for (int b = 0; b < 2; ++b) {
         if (b == 1 && !has_q1) break;
-        // own-chunk token mask (masked instance): this thread's 64 bits of its
-        // row, fetched before the wait so that the load hides behind it
-        const bool own_tile = kOwn && kt < p.nt_slot;
+        // token-level mask (token-mask instance): this thread's 64 bits of its
+        // row for this key tile, from the own-chunk mask or from the history
+        // mask of the tile's key state (the caller's context index); fetched
+        // before the wait so that the load hides behind it
+        const int kst = kOwn ? kt / p.nt_slot : 0;  // key state: 0 own, then the visible contexts
+        const bool own_tile = kOwn && (kst == 0 ? p.own_mask : p.hist_mask) != nullptr;
         uint32_t ow[2] = {~0u, ~0u};
         if (own_tile) {
           const int u = (qt0 + b) * kTile + row;
           if (u < p.T) {  // rows past T are never stored
-            const uint32_t* mrow = p.own_mask + ((size_t)nd.q_index * p.T + u) * p.own_words;
-            const int wi = kt * 4 + half * 2;  // word holding key 128 kt + 64 half
-            ow[0] = wi < p.own_words ? __ldg(mrow + wi) : 0u;
-            ow[1] = wi + 1 < p.own_words ? __ldg(mrow + wi + 1) : 0u;
+            const size_t qrow = (size_t)nd.q_index * p.T + u;
+            const uint32_t* mrow =
+                kst == 0 ? p.own_mask + qrow * p.own_words
+                         : p.hist_mask + (qrow * p.hist_states + (nd.src[kst] - 1)) * p.hist_words;
+            const int words = kst == 0 ? p.own_words : p.hist_words;
+            const int wi = (kt - kst * p.nt_slot) * 4 + half * 2;  // key 128 t + 64 half of the state
+            ow[0] = wi < words ? __ldg(mrow + wi) : 0u;
+            ow[1] = wi + 1 < words ? __ldg(mrow + wi + 1) : 0u;
           }
         }
         ok = mbar_wait(&bars.s_full[b], (uint32_t)i & 1u, &abort_flag, tmo);
@@ -885,7 +892,7 @@ cudaError_t launch_d(const AttnParams& p, int grid, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   e = configure_d<D>(dev);
   if (e != cudaSuccess) return e;
-  if (p.masked && p.own_mask != nullptr)
+  if (p.masked && (p.own_mask != nullptr || p.hist_mask != nullptr))
     attend_kernel<D, true, true><<<grid, kThreads, C::kSmemBytes, s>>>(p);
   else if (p.masked)
     attend_kernel<D, true, false><<<grid, kThreads, C::kSmemBytes, s>>>(p);

@@ -59,7 +59,12 @@ struct alignas(128) AttnParams {
   int32_t mask_words;
   const uint32_t* own_mask;   // token visibility in the own chunk [n_nodes][T][own_words], or null
   int32_t own_words;
-  int32_t masked;             // tile_mask or own_mask given: the masked kernel instance
+  // token visibility of the context states [n_nodes][T][hist_states][hist_words]
+  // (state j = the caller's ctx_slot[j]), or null
+  const uint32_t* hist_mask;
+  int32_t hist_states;
+  int32_t hist_words;
+  int32_t masked;             // a tile or token mask given: a masked kernel instance
   AttnNode nodes[SVA_MAX_NODES];
 };
 

@@ -629,11 +629,13 @@ enum class Scratch {
 };
 
 // sva_attend_nodes, _sparse, _masked and _noalloc: the checks, the launch
-// parameters, the split plan and the launch.  tile_mask and own_mask NULL is
+// parameters, the split plan and the launch.  tile_mask, own_mask and
+// hist_mask NULL is
 // the dense mask.  Every check runs before anything is enqueued.
 sva_status attend(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* q, void* out,
                   float* lse, float scale, const uint32_t* tile_mask, int32_t mask_words,
-                  const uint32_t* own_mask, int32_t own_words, sva_stream s, Scratch scratch) {
+                  const uint32_t* own_mask, int32_t own_words, const uint32_t* hist_mask,
+                  int32_t hist_states, int32_t hist_words, sva_stream s, Scratch scratch) {
   if (c == nullptr || nodes == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "NULL argument");
   if (n_nodes < 1) return fail(SVA_ERR_INVALID_ARGUMENT, "n_nodes %d < 1", n_nodes);
   if (n_nodes > SVA_MAX_NODES)
@@ -715,7 +717,23 @@ sva_status attend(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const vo
     p.own_mask = own_mask;
     p.own_words = own_words;
   }
-  p.masked = (tile_mask != nullptr || own_mask != nullptr) ? 1 : 0;
+  if (hist_mask != nullptr) {
+    if ((reinterpret_cast<uintptr_t>(hist_mask) & 3u) != 0)
+      return fail(SVA_ERR_INVALID_ARGUMENT, "hist_mask must be 4-byte aligned");
+    if (hist_words < (c->L.T + 31) / 32)
+      return fail(SVA_ERR_INVALID_ARGUMENT, "hist_words %d < %d needed for %d tokens", hist_words,
+                  (c->L.T + 31) / 32, c->L.T);
+    if (hist_states < 1)
+      return fail(SVA_ERR_INVALID_ARGUMENT, "hist_states %d < 1", hist_states);
+    for (int i = 0; i < n_nodes; ++i)
+      if (nodes[i].n_ctx > hist_states)
+        return fail(SVA_ERR_INVALID_ARGUMENT, "node %d has %d context states, hist_states is %d",
+                    i, nodes[i].n_ctx, hist_states);
+    p.hist_mask = hist_mask;
+    p.hist_states = hist_states;
+    p.hist_words = hist_words;
+  }
+  p.masked = (tile_mask != nullptr || own_mask != nullptr || hist_mask != nullptr) ? 1 : 0;
   if (p.masked)  // the masked kernel keeps a bitmap of the node's key tiles
     for (int i = 0; i < n_nodes; ++i)
       if ((long long)p.nodes[i].n_kv * p.nt_slot > 32LL * sva::kMaskWords)
@@ -803,7 +821,7 @@ extern "C" {
 
 sva_status sva_attend_nodes(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const void* q,
                             void* out, float* lse, float scale, sva_stream s) {
-  return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, s,
+  return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, nullptr, 0, 0, s,
                 Scratch::kWorkspace);
 }
 
@@ -964,18 +982,19 @@ sva_status sva_attend_nodes_sparse(sva_cache* c, const sva_node* nodes, int32_t 
                                    const uint32_t* tile_mask, int32_t words_per_row,
                                    sva_stream s) {
   if (tile_mask == nullptr) return fail(SVA_ERR_INVALID_ARGUMENT, "tile_mask is NULL");
-  return attend(c, nodes, n_nodes, q, out, lse, scale, tile_mask, words_per_row, nullptr, 0, s,
-                Scratch::kWorkspace);
+  return attend(c, nodes, n_nodes, q, out, lse, scale, tile_mask, words_per_row, nullptr, 0,
+                nullptr, 0, 0, s, Scratch::kWorkspace);
 }
 
 sva_status sva_attend_nodes_masked(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
                                    const void* q, void* out, float* lse, float scale,
                                    const sva_attn_mask* mask, sva_stream s) {
   if (mask == nullptr)
-    return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, s,
+    return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, nullptr, 0, 0, s,
                   Scratch::kWorkspace);
   return attend(c, nodes, n_nodes, q, out, lse, scale, mask->tile_mask, mask->tile_words,
-                mask->own_mask, mask->own_words, s, Scratch::kWorkspace);
+                mask->own_mask, mask->own_words, mask->hist_mask, mask->hist_states,
+                mask->hist_words, s, Scratch::kWorkspace);
 }
 
 // Attention with the split scratch taken from the library's own device
@@ -985,7 +1004,7 @@ sva_status sva_attend_nodes_masked(sva_cache* c, const sva_node* nodes, int32_t 
 sva_status sva_attend_nodes_noalloc(sva_cache* c, const sva_node* nodes, int32_t n_nodes,
                                     const void* q, void* out, float* lse, float scale,
                                     sva_stream s) {
-  return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, s,
+  return attend(c, nodes, n_nodes, q, out, lse, scale, nullptr, 0, nullptr, 0, nullptr, 0, 0, s,
                 Scratch::kStatic);
 }
 

@@ -255,6 +255,44 @@ def own_mask(w: Workload, density: float, seed: int | None = None) -> torch.Tens
     return pack_bits(keep, -(-w.T // 32))
 
 
+def _splitmix64(x):
+    """splitmix64 (Steele, Lea and Flood, 2014) of uint64 numpy values."""
+    import numpy as np
+    x = (x + np.uint64(0x9E3779B97F4A7C15)) & np.uint64(0xFFFFFFFFFFFFFFFF)
+    z = x
+    z = ((z ^ (z >> np.uint64(30))) * np.uint64(0xBF58476D1CE4E5B9)) & np.uint64(0xFFFFFFFFFFFFFFFF)
+    z = ((z ^ (z >> np.uint64(27))) * np.uint64(0x94D049BB133111EB)) & np.uint64(0xFFFFFFFFFFFFFFFF)
+    return z ^ (z >> np.uint64(31))
+
+
+def hist_mask(w: Workload, density: float, seed: int | None = None) -> torch.Tensor:
+    """Seeded token-level visibility of the history, int32
+    [n_nodes][T][W][ceil(T/32)] words: bit v of row (node i, query u,
+    context j) is kept when a counter-based uniform, splitmix64 of the index
+    (((seed * n + i) * W + j) * T + u) * T + v scaled to [0, 1), is below
+    `density` (default seed: the workload's seed + 4000); row 7 of every
+    node sees no history key.  Context j is the node's j-th selected state;
+    rows past a node's context count are drawn too and ignored.  Counter
+    based, so a large workload's mask needs no stream of draws."""
+    import numpy as np
+    seed = w.seed + 4000 if seed is None else seed
+    T, W, n = w.T, w.W, w.n_nodes
+    words = -(-T // 32)
+    out = np.empty((n, T, W, words), dtype="<i4")
+    v = np.arange(T, dtype=np.uint64)
+    u = np.arange(T, dtype=np.uint64)[:, None]
+    cut = np.uint64(int(density * 2.0 ** 64) if density < 1.0 else 2 ** 64 - 1)
+    for i in range(n):
+        for j in range(W):
+            base = np.uint64((((seed * n + i) * W + j) * T) * T)
+            keep = _splitmix64(base + u * np.uint64(T) + v[None, :]) < cut
+            if density >= 1.0:
+                keep[:] = True
+            keep[7 % T, :] = False
+            out[i, :, j, :] = pack_bits(keep, words).numpy()
+    return torch.from_numpy(out)
+
+
 def pack_bits(keep: torch.Tensor, words: int) -> torch.Tensor:
     """bool [..., nbits] -> int32 [..., words], bit k in word k // 32 at position k % 32."""
     import numpy as np

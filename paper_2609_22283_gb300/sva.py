@@ -67,7 +67,9 @@ class sva_node(ctypes.Structure):
 
 class sva_attn_mask(ctypes.Structure):
     _fields_ = [("tile_mask", ctypes.c_void_p), ("tile_words", ctypes.c_int32),
-                ("own_mask", ctypes.c_void_p), ("own_words", ctypes.c_int32)]
+                ("own_mask", ctypes.c_void_p), ("own_words", ctypes.c_int32),
+                ("hist_mask", ctypes.c_void_p), ("hist_states", ctypes.c_int32),
+                ("hist_words", ctypes.c_int32)]
 
 
 _lib = None
@@ -323,10 +325,11 @@ class Cache:
         _check(st)
 
     def attend_nodes_masked(self, nodes, q, out, lse=None, scale=None, tile_mask=None,
-                            own_mask=None, stream=None, check=True):
+                            own_mask=None, hist_mask=None, stream=None, check=True):
         """sva_attend_nodes_masked: tile_mask as in attend_nodes_sparse, own_mask a
-        contiguous int32 CUDA tensor [n_nodes][T][words] of own-chunk token bits;
-        either may be None."""
+        contiguous int32 CUDA tensor [n_nodes][T][words] of own-chunk token bits,
+        hist_mask one [n_nodes][T][states][words] of history token bits (state
+        j = the node's j-th context); any may be None."""
         n = len(nodes) if not isinstance(nodes, ctypes.Array) else None
         arr = nodes if isinstance(nodes, ctypes.Array) else make_nodes(nodes)
         count = n if n is not None else len(arr)
@@ -338,10 +341,17 @@ class Cache:
             if t is not None and (t.dtype != torch.int32 or not t.is_cuda or not t.is_contiguous()
                                   or t.dim() != 3 or tuple(t.shape[:2]) != (count, rows)):
                 raise ValueError(f"{nm} must be a contiguous int32 CUDA tensor [{count}][{rows}][words]")
+        if hist_mask is not None and (hist_mask.dtype != torch.int32 or not hist_mask.is_cuda
+                                      or not hist_mask.is_contiguous() or hist_mask.dim() != 4
+                                      or tuple(hist_mask.shape[:2]) != (count, self.T)):
+            raise ValueError(f"hist_mask must be a contiguous int32 CUDA tensor [{count}][{self.T}][states][words]")
         m = sva_attn_mask(ctypes.c_void_p(tile_mask.data_ptr() if tile_mask is not None else 0),
                           int(tile_mask.shape[2]) if tile_mask is not None else 0,
                           ctypes.c_void_p(own_mask.data_ptr() if own_mask is not None else 0),
-                          int(own_mask.shape[2]) if own_mask is not None else 0)
+                          int(own_mask.shape[2]) if own_mask is not None else 0,
+                          ctypes.c_void_p(hist_mask.data_ptr() if hist_mask is not None else 0),
+                          int(hist_mask.shape[2]) if hist_mask is not None else 0,
+                          int(hist_mask.shape[3]) if hist_mask is not None else 0)
         if scale is None:
             scale = 1.0 / math.sqrt(g.head_dim)
         st = _lib.sva_attend_nodes_masked(self.handle, arr, count, ctypes.c_void_p(q.data_ptr()),

@@ -70,13 +70,13 @@ def oracle_masks(w: I.Workload, mask=None) -> np.ndarray:
 
 
 def oracle_node(w, inp, states, node_index, heads, rows, hidden=frozenset(), tile_mask=None,
-                own_mask=None):
+                own_mask=None, hist_mask=None):
     g = oracle_geometry(w)
     q = inp.q[node_index].float().numpy()
     out, lse, _ = oracle.node_forward(g, oracle.POLICY_IDS[w.policy], w.W, w.nodes[node_index],
                                       states, q, list(heads), list(rows), 1.0 / math.sqrt(w.d),
                                       hidden=hidden, within=w.within, tile_mask=tile_mask,
-                                      own_mask=own_mask,
+                                      own_mask=own_mask, hist_mask=hist_mask,
                                       norm=((inp.gamma_k.double().numpy(), inp.gamma_q.double().numpy(),
                                              inp.norm_eps) if w.qknorm else None))
     return out, lse
