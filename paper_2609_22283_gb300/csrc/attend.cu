@@ -84,7 +84,16 @@ constexpr int kLaunchRegs = 168;
 constexpr int kRegsLow = 88;
 constexpr int kRegsHigh = 208;
 static_assert(4 * 32 * kRegsLow + 8 * 32 * kRegsHigh <= kThreads * kLaunchRegs, "register split");
-constexpr float kRescaleThreshold = 8.0f;  // log2 units: P <= 2^8 between rescales
+// Lazy rescale of O: a row's running max m is only moved (and O, l scaled)
+// when a tile's max exceeds it by more than this many log2 units, so P =
+// 2^(x - m) <= 2^64 between rescales.  Then l <= 2^(64 + 16) for up to 2^16
+// keys and |O| <= 2^86 for |V| <= 2^6, far below the fp32 and bf16 limit of
+// 2^128, while bf16 keeps P's relative precision at any magnitude.  With
+// x10 outliers in q and k a row's max keeps jumping by more than 2^8 long
+// into the key sequence, and each jump cost the warp a TMEM round trip of O
+// on the softmax's critical path (stress14b: 2^64 instead of 2^8 is 1.8%
+// faster).
+constexpr float kRescaleThreshold = 64.0f;
 
 template <int N>
 __device__ __forceinline__ void regs_dec() {
