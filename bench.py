@@ -94,6 +94,19 @@ def attn_flops(w) -> float:
     return total
 
 
+def attn_bytes(w) -> float:
+    """Algorithmic DRAM bytes of one attention launch: the K and V of every
+    distinct state the nodes read (once per head), Q read and O written once."""
+    read = set()
+    for (s, b, j) in w.nodes:
+        read.add((s, b, j))
+        for r in range(1, max(0, min(w.W, b - 1)) + 1):
+            lvl = 0 if w.policy == "clean" else (j if w.policy == "same" else max(j - r, 0))
+            read.add((s, b - r, lvl))
+    kv = len(read) * 2 * w.H * w.T * w.d * 2.0
+    return kv + 2 * w.n_nodes * w.T * w.H * w.d * 2.0
+
+
 def rope_bytes(w) -> float:
     """Algorithmic bytes of one rope_kv_write launch: K, V, Q read once, written once."""
     return 3 * 2 * w.n_nodes * w.T * w.H * w.d * 2.0
@@ -504,7 +517,11 @@ def run_ours(args, world, rank, local):
                      "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
                      "peak_source": f"{peak_src} bf16 dense burst (MEASURED_PEAKS.json)"
                      if peak_src == "measured" else "fallback 1.9 PFLOP/s",
-                     "traffic": traffic},
+                     "traffic": traffic,
+                     "algorithmic_bytes": attn_bytes(w),
+                     # context: the cuBLAS loop measured under the power cap
+                     "frac_of_sustained": achieved / peaks.get(
+                         "bf16_tflops_sustained", FALLBACK_PEAKS["bf16_tflops_sustained"])},
         "e2e": {"value": flops * world / (e2e_step * 1e-3) / 1e12, "unit": "TFLOP/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": e2e_step, "steps": k_e2e,

@@ -40,3 +40,15 @@ def test_frame_causal_counts():
     per_node = [4.0 * (32 * (32 + 64 + 96) + 96 * max(0, min(t.W, b - 1)) * 96) * t.d * t.H
                 for (_, b, _) in t.nodes]
     assert bench.attn_flops(t) == sum(per_node)
+
+
+def test_attention_algorithmic_bytes():
+    # distinct states read x (K + V) x heads x T x d x 2 B, plus Q read and O written
+    slot = 2 * 4680 * 128 * 2
+    assert bench.attn_bytes(I.WORKLOADS["clean1"]) == 4 * 12 * slot + 2 * 1 * 12 * 4680 * 128 * 2
+    # prog4: the 4 nodes' own states and the clean chunks 11..16 (10 states)
+    assert bench.attn_bytes(I.WORKLOADS["prog4"]) == 10 * 12 * slot + 2 * 4 * 12 * 4680 * 128 * 2
+    # stress14b: two streams of prog4's states, 40 heads
+    assert bench.attn_bytes(I.WORKLOADS["stress14b"]) == 20 * 40 * slot + 2 * 8 * 40 * 4680 * 128 * 2
+    # same4: each node's own state and its three same-level predecessors
+    assert bench.attn_bytes(I.WORKLOADS["same4"]) == 16 * 12 * slot + 2 * 4 * 12 * 4680 * 128 * 2
