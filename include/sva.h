@@ -13,8 +13,9 @@
  * (Eq. 4).  Several nodes of one pipeline round (Eq. 6) are processed by one
  * launch, which is how progressive history is executed (Section 3.3).
  * Around that: the input projection producing q, k, v (sva_qkv_project), the
- * RoPE + cache write (sva_rope_kv_write), and a block-sparse form of the
- * token mask of Eq. 4 (sva_attend_nodes_sparse).
+ * RoPE + cache write (sva_rope_kv_write), a block-sparse form of the token
+ * mask of Eq. 4 (sva_attend_nodes_sparse) and its token-level form on the
+ * own chunk and on the history (sva_attend_nodes_masked).
  *
  * Conventions shared by every entry point
  * ---------------------------------------
