@@ -97,6 +97,9 @@ struct ProjParams {
   CUtensorMap tmap_x;   // x as 2D (C, rows), box (64, 128), 128B swizzle
   CUtensorMap tmap_w;   // weight as 2D (C, 3N), box (64, BN), 128B swizzle
   CUtensorMap tmap_wh;  // the same weight with box (64, BN / 2): half-width items
+  // out[i] as 2D (N, rows), box (32, 32), 64B swizzle: the epilogue's tile
+  // stores (with rope_on only tmap_out[0], Q' token-major)
+  CUtensorMap tmap_out[3];
   const float* bias;    // [3N] fp32, or null
   void* out[3];         // q, k, v: bf16 [rows][N]
   int* status;          // device status word

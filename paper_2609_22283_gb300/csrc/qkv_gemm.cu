@@ -20,14 +20,19 @@
 //   warp 1      TMEM owner and MMA issuer (whole warp, one elected lane);
 //   warps 4-11  epilogue: two warps per TMEM lane quarter, one output row per
 //               thread, the two warps of a quarter taking alternate 32-column
-//               chunks.
+//               chunks.  Each chunk (32 rows x 64 bytes) is staged in the
+//               warp's shared-memory buffers and leaves by one TMA tile store
+//               (two buffers per warp, reused once the store has read them):
+//               a per-thread store would touch 32 rows per warp instruction.
 // An item never straddles q, k and v (N is a multiple of BN), so its epilogue
 // writes into one tensor.  With the fused RoPE epilogue (sva_qkv_project_rope)
 // each thread rotates the pairs of its row's q and k columns in fp32 at the
-// token's (t, h, w) position before the one bf16 rounding, writes Q' token-
-// major and scatters K' and V into the node's own cache slot.  Rows past
-// `rows` read zeros (TMA fill) and are not stored; K past C reads zeros on
-// both operands.  All waits are bounded: on expiry the CTA records
+// token's (t, h, w) position before the one bf16 rounding; Q' leaves token-
+// major by tile store, K' and V are scattered into the node's own cache slot
+// by the warp reading the staged chunk back, eight whole 64-byte cache rows
+// per store instruction (the rows of a chunk may belong to two nodes).  Rows
+// past `rows` read zeros (TMA fill) and are not stored; K past C reads zeros
+// on both operands.  All waits are bounded: on expiry the CTA records
 // SVA_ERR_DEVICE_TIMEOUT, drains its own copies and MMAs, frees TMEM and
 // exits.
 #include <mutex>
@@ -48,13 +53,15 @@ constexpr int kStages = 4;
 constexpr int kBM = 128;
 constexpr int kBK = 64;
 constexpr int kEpiWarps = 8;
+constexpr int kChunkBytes = 32 * 64;  // one staged 32 x 32 bf16 output chunk
 
 template <int BN>
 struct ProjCfg {
   static constexpr int kABytes = kBM * kBK * 2;  // 16 KB
   static constexpr int kBBytes = BN * kBK * 2;   // 32 KB at BN = 256
   static constexpr int kStageBytes = kABytes + kBBytes;
-  static constexpr int kSmemBytes = kStages * kStageBytes + 1024;  // + alignment slack
+  static constexpr int kOutBytes = kEpiWarps * 2 * kChunkBytes;  // output staging, 32 KB
+  static constexpr int kSmemBytes = kStages * kStageBytes + kOutBytes + 1024;  // + alignment slack
   static constexpr uint32_t kTmemCols = 2 * BN;                   // two accumulators
 };
 
@@ -213,37 +220,77 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
     const int part = (warp - 4) >> 2;  // which alternate 32-column chunks
     const int row = q4 * 32 + lane;
     const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
+    // This warp's two staging buffers.  A chunk is 32 rows (one per lane) of
+    // 64 bytes; 16-byte piece j of row r sits at piece j ^ ((r >> 1) & 3) (the
+    // 64-byte swizzle of the output tensor maps), so that the eight lanes of
+    // a shared-memory phase, four row pairs, hit 32 different banks.
+    const uint32_t stage0 =
+        smem_u32(smem + kStages * C::kStageBytes) + (uint32_t)((warp - 4) * 2 * kChunkBytes);
+    int staged = 0;  // chunks this warp has staged
+    // This lane's row of a chunk (16 words) into the next buffer, once the
+    // bulk store that last read that buffer is done with it; a chunk that
+    // will not leave by a bulk store first lets every such store finish
+    // reading, whichever buffer it came from.
+    auto stage = [&](const uint32_t (&w)[16], bool bulk) -> uint32_t {
+      const uint32_t buf = stage0 + (uint32_t)((staged & 1) * kChunkBytes);
+      ++staged;
+      if (lane == 0) {
+        if (bulk)
+          bulk_wait_group_read<1>();
+        else
+          bulk_wait_group_read<0>();
+      }
+      __syncwarp();
+      const uint32_t at = buf + (uint32_t)(lane * 64);
+      const int sw = (lane >> 1) & 3;
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        st_shared_v4(at + (uint32_t)((j ^ sw) << 4), w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
+      return buf;
+    };
+    // A staged chunk to global by one bulk tensor store: columns [x, x + 32)
+    // of rows [y, y + 32) of the map's tensor (rows past its extent are not
+    // written).
+    auto store_tile = [&](uint32_t buf, const CUtensorMap* map, int x, int y) {
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0 && y < p.rows) {
+        tma_store_2d(map, buf, x, y);
+        bulk_commit_group();
+      }
+    };
+    // A staged chunk to rows scattered in the cache: row j * 8 + lane / 4 to
+    // rowp[j] + off (rows with a null pointer are skipped); four lanes per
+    // 64-byte row, eight whole rows per store instruction.
+    auto store_rows = [&](uint32_t buf, const uint64_t (&rowp)[4], size_t off) {
+      __syncwarp();
+      const int piece = lane & 3;
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const int r = j * 8 + (lane >> 2);
+        const uint4 v = ld_shared_v4(buf + (uint32_t)(r * 64 + ((piece ^ ((r >> 1) & 3)) << 4)));
+        if (rowp[j] != 0)
+          *reinterpret_cast<uint4*>(reinterpret_cast<__nv_bfloat16*>(rowp[j]) + off + piece * 8) = v;
+      }
+    };
     bool ok = true;
     int tc = 0;
     for (int i = blockIdx.x; ok && i < p.n_items; i += gridDim.x, ++tc) {
       const Item it = item_of(p, i);
       const int width = it.half >= 0 ? BN / 2 : BN;  // output columns of this item
       const int acc = tc & 1;
-      ok = mbar_wait(&bars.acc_full[acc], (uint32_t)(tc >> 1) & 1u, &abort_flag, tmo);
-      ok = __all_sync(0xffffffffu, ok);
-      if (!ok) break;
-      tc_fence_after();
+      // Waits for this item's accumulator; what depends only on the item is
+      // worked out (and fetched) before, while the MMAs still run.
+      auto wait_acc = [&]() {
+        const bool got = __all_sync(0xffffffffu, mbar_wait(&bars.acc_full[acc], (uint32_t)(tc >> 1) & 1u,
+                                                            &abort_flag, tmo));
+        tc_fence_after();
+        return got;
+      };
       const int col = it.n * BN + (it.half > 0 ? BN / 2 : 0);  // output column in [0, 3N)
       const int tensor = col / p.N;      // q, k or v
       const int c0 = col - tensor * p.N;  // column inside that tensor
-      const long long grow = (long long)it.m * kBM + row;
-      const bool in_range = grow < p.rows;
-      __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.out[p.rope_on ? 0 : tensor]) + grow * p.N + c0;
-      // fused RoPE: this row's node, token and position, and where K' / V go
-      int tpos = 0, hh = 0, ww = 0;
-      __nv_bfloat16* cdst = nullptr;  // (slot, K or V, head 0, token u, dim 0) of the cache
-      if (p.rope_on && in_range) {
-        const RopeParams& rp = p.rope;
-        const int node = (int)(grow / rp.T);
-        const int u = (int)(grow - (long long)node * rp.T);
-        const int HpWp = rp.Hp * rp.Wp;
-        const int f = u / HpWp;
-        hh = (u - f * HpWp) / rp.Wp;
-        ww = u - f * HpWp - hh * rp.Wp;
-        tpos = rp.nodes[node].t_base + f;
-        cdst = static_cast<__nv_bfloat16*>(rp.cache) +
-               ((((size_t)rp.nodes[node].slot * 2 + (tensor == 2 ? 1 : 0)) * rp.H) * rp.Tpad + u) * rp.d;
-      }
+      const int y0 = it.m * kBM + q4 * 32;  // first output row of this warp
       // 32 accumulator columns of this row: TMEM -> registers, plus the bias
       auto load_chunk = [&](int c, uint32_t (&r)[32], float (&bv)[32]) {
         tmem_ld32(tbase + lane_off + (uint32_t)(acc * BN + c * 32), r);
@@ -261,16 +308,35 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
         }
       };
       if (p.rope_on) {
-        // Fused RoPE: the 32-column chunk ci of every head in the item uses
-        // the same 16 (cos, sin) pairs, fetched once per chunk index (the
-        // next one while the current one is rotated); this warp takes the
-        // chunk indices of its parity.  Pairs [0, P0) rotate with the frame
-        // index, [P0, P0+P1) with the patch row, the rest with the patch
-        // column (the values and split of the RoPE + cache write); the
-        // patch-row and patch-column tables here are the pair-major copies,
-        // so the 32 tokens of a warp read neighbouring entries.  An item
-        // covers whole heads (the host splits a tile only when its halves do).
+        // Fused RoPE: this row's node, token and position, and where K' / V go
         const RopeParams& rp = p.rope;
+        const long long grow = (long long)it.m * kBM + row;
+        int tpos = 0, hh = 0, ww = 0;
+        uint64_t cdst = 0;  // (slot, K or V, head 0, token u, dim 0) of the cache; 0 past `rows`
+        if (grow < p.rows) {
+          const int node = (int)(grow / rp.T);
+          const int u = (int)(grow - (long long)node * rp.T);
+          const int HpWp = rp.Hp * rp.Wp;
+          const int f = u / HpWp;
+          hh = (u - f * HpWp) / rp.Wp;
+          ww = u - f * HpWp - hh * rp.Wp;
+          tpos = rp.nodes[node].t_base + f;
+          cdst = reinterpret_cast<uint64_t>(
+              static_cast<__nv_bfloat16*>(rp.cache) +
+              ((((size_t)rp.nodes[node].slot * 2 + (tensor == 2 ? 1 : 0)) * rp.H) * rp.Tpad + u) * rp.d);
+        }
+        uint64_t rowp[4];  // the cache rows this lane writes in store_rows
+#pragma unroll
+        for (int j = 0; j < 4; ++j) rowp[j] = __shfl_sync(0xffffffffu, cdst, j * 8 + (lane >> 2));
+        // The 32-column chunk ci of every head in the item uses the same 16
+        // (cos, sin) pairs, fetched once per chunk index (the next one while
+        // the current one is rotated); this warp takes the chunk indices of
+        // its parity.  Pairs [0, P0) rotate with the frame index, [P0, P0+P1)
+        // with the patch row, the rest with the patch column (the values and
+        // split of the RoPE + cache write); the patch-row and patch-column
+        // tables here are the pair-major copies, so the 32 tokens of a warp
+        // read neighbouring entries.  An item covers whole heads (the host
+        // splits a tile only when its halves do).
         const int cpd = rp.d / 32;  // chunks per head (even: d is 64 or 128)
         const int heads = width / rp.d;
         const float2* pt = rp.tab_t + (size_t)tpos * rp.P0;  // this token's frame row
@@ -287,6 +353,8 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
         };
         float2 cs_next[16];
         if (tensor != 2) load_cs(part, cs_next);
+        ok = wait_acc();
+        if (!ok) break;
 #pragma unroll 1
         for (int ci = part; ci < cpd; ci += 2) {
           float2 cs[16];
@@ -299,44 +367,38 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
             uint32_t r[32];
             float bv[32];
             load_chunk(c, r, bv);  // warp-collective: every thread, in range or not
-            if (in_range) {
+            uint32_t w[16];
+            if (tensor == 2) {
+#pragma unroll
+              for (int e = 0; e < 16; ++e)
+                w[e] = pack2_bf16(__uint_as_float(r[2 * e]) + bv[2 * e], __uint_as_float(r[2 * e + 1]) + bv[2 * e + 1]);
+            } else {
+#pragma unroll
+              for (int e = 0; e < 16; ++e)
+                w[e] = rotate2_bf16(__uint_as_float(r[2 * e]) + bv[2 * e],
+                                    __uint_as_float(r[2 * e + 1]) + bv[2 * e + 1], cs[e]);
+            }
+            if (tensor == 0) {
+              store_tile(stage(w, true), &p.tmap_out[0], c0 + c * 32, y0);  // Q' token-major
+            } else {
               const int head = (c0 + c * 32) / rp.d;
-              uint32_t w[16];
-              if (tensor == 2) {
-#pragma unroll
-                for (int e = 0; e < 16; ++e)
-                  w[e] = pack2_bf16(__uint_as_float(r[2 * e]) + bv[2 * e], __uint_as_float(r[2 * e + 1]) + bv[2 * e + 1]);
-              } else {
-#pragma unroll
-                for (int e = 0; e < 16; ++e)
-                  w[e] = rotate2_bf16(__uint_as_float(r[2 * e]) + bv[2 * e],
-                                      __uint_as_float(r[2 * e + 1]) + bv[2 * e + 1], cs[e]);
-              }
-              uint4* d4 = reinterpret_cast<uint4*>(
-                  tensor == 0 ? dst + c * 32 : cdst + (size_t)head * rp.Tpad * rp.d + ci * 32);
-#pragma unroll
-              for (int v = 0; v < 4; ++v) d4[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
+              store_rows(stage(w, false), rowp, (size_t)head * rp.Tpad * rp.d + (size_t)ci * 32);
             }
           }
         }
       } else {
+        ok = wait_acc();
+        if (!ok) break;
 #pragma unroll 1
         for (int c = part; c < width / 32; c += 2) {
           uint32_t r[32];
           float bv[32];
           load_chunk(c, r, bv);  // warp-collective: every thread, in range or not
-          if (in_range) {
-            uint4* d4 = reinterpret_cast<uint4*>(dst + c * 32);
+          uint32_t w[16];
 #pragma unroll
-            for (int v = 0; v < 4; ++v) {
-              uint4 w;
-              w.x = pack2_bf16(__uint_as_float(r[8 * v + 0]) + bv[8 * v + 0], __uint_as_float(r[8 * v + 1]) + bv[8 * v + 1]);
-              w.y = pack2_bf16(__uint_as_float(r[8 * v + 2]) + bv[8 * v + 2], __uint_as_float(r[8 * v + 3]) + bv[8 * v + 3]);
-              w.z = pack2_bf16(__uint_as_float(r[8 * v + 4]) + bv[8 * v + 4], __uint_as_float(r[8 * v + 5]) + bv[8 * v + 5]);
-              w.w = pack2_bf16(__uint_as_float(r[8 * v + 6]) + bv[8 * v + 6], __uint_as_float(r[8 * v + 7]) + bv[8 * v + 7]);
-              d4[v] = w;
-            }
-          }
+          for (int e = 0; e < 16; ++e)
+            w[e] = pack2_bf16(__uint_as_float(r[2 * e]) + bv[2 * e], __uint_as_float(r[2 * e + 1]) + bv[2 * e + 1]);
+          store_tile(stage(w, true), &p.tmap_out[tensor], c0 + c * 32, y0);
         }
       }
       // The MMA warp may overwrite this accumulator once every epilogue warp
@@ -345,6 +407,10 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
       __syncwarp();
       if (lane == 0) mbar_arrive(&bars.acc_empty[acc]);
     }
+    // the bulk stores read this CTA's shared memory and must be complete
+    // before it exits
+    if (lane == 0) bulk_wait_group<0>();
+    __syncwarp();
     if (!ok) proj_timeout(p, &abort_flag);
   }
 

@@ -889,6 +889,21 @@ sva_status project(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const v
     if (r != CUDA_SUCCESS)
       return fail(SVA_ERR_CUDA, "cuTensorMapEncodeTiled(weight) failed: %d", (int)r);
   }
+  {
+    // the epilogue's tile stores: 32 rows x 32 columns (64 bytes), staged in
+    // shared memory in the 64-byte swizzle; rows past `rows` are not written
+    void* outs[3] = {q, k, v};
+    for (int i = 0; i < (rope ? 1 : 3); ++i) {
+      cuuint64_t dims[2] = {(cuuint64_t)N, (cuuint64_t)rows};
+      cuuint64_t strides[1] = {(cuuint64_t)N * 2};
+      cuuint32_t box[2] = {32, 32};
+      CUresult r = fn(&p.tmap_out[i], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, outs[i], dims, strides,
+                      box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+                      CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      if (r != CUDA_SUCCESS)
+        return fail(SVA_ERR_CUDA, "cuTensorMapEncodeTiled(output %d) failed: %d", i, (int)r);
+    }
+  }
   if (rope) {
     // the same node checks as sva_rope_kv_write
     for (int i = 0; i < n_nodes; ++i) {
