@@ -18,7 +18,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libsva.so")
 
 SOURCES = ["attend.cu", "attend_noalloc.cu", "rope_kv.cu", "qkv_gemm.cu", "sva_api.cpp"]
-HEADERS = [os.path.join(CSRC, h) for h in ("internal.h", "ptx.cuh")] + [os.path.join(INCLUDE, "sva.h")]
+HEADERS = [os.path.join(CSRC, h) for h in ("internal.h", "proj.h", "ptx.cuh")] + [os.path.join(INCLUDE, "sva.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-lineinfo", "-O3", "-std=c++17", "-Xcompiler", "-fPIC",
                      "-I" + INCLUDE, "-I" + CSRC]

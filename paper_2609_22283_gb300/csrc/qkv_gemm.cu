@@ -41,6 +41,7 @@
 #include <cuda_runtime.h>
 
 #include "internal.h"
+#include "proj.h"
 #include "ptx.cuh"
 
 namespace sva {

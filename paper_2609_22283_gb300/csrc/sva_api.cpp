@@ -21,6 +21,7 @@
 #include <cuda_runtime.h>
 
 #include "internal.h"
+#include "proj.h"
 #include "sva.h"
 
 namespace {
