@@ -12,7 +12,9 @@ struct ProjParams {
   CUtensorMap tmap_w;   // weight as 2D (C, 3N), box (64, BN), 128B swizzle
   CUtensorMap tmap_wh;  // the same weight with box (64, BN / 2): half-width items
   // out[i] as 2D (N, rows), box (32, 32), 64B swizzle: the epilogue's tile
-  // stores (with rope_on only tmap_out[0], Q' token-major)
+  // stores.  With rope_on: tmap_out[0] is Q' token-major, tmap_out[1] the
+  // slot pool as 3D (d, T, num_slots * 2 * H) with the (slot, K|V, head)
+  // stride Tpad * d, box (32, 32, 1), so that rows past T are not written.
   CUtensorMap tmap_out[3];
   const float* bias;    // [3N] fp32, or null
   void* out[3];         // q, k, v: bf16 [rows][N]

@@ -28,11 +28,12 @@
 // writes into one tensor.  With the fused RoPE epilogue (sva_qkv_project_rope)
 // each thread rotates the pairs of its row's q and k columns in fp32 at the
 // token's (t, h, w) position before the one bf16 rounding; Q' leaves token-
-// major by tile store, K' and V are scattered into the node's own cache slot
-// by the warp reading the staged chunk back, eight whole 64-byte cache rows
-// per store instruction (the rows of a chunk may belong to two nodes).  Rows
-// past `rows` read zeros (TMA fill) and are not stored; K past C reads zeros
-// on both operands.  All waits are bounded: on expiry the CTA records
+// major by tile store, K' and V by tile stores into the node's own cache
+// slot (a 3D map of the slot pool that clips rows past T); a chunk whose 32
+// rows belong to two nodes is scattered by the warp reading it back, eight
+// whole 64-byte cache rows per store instruction.  Rows past `rows` read
+// zeros (TMA fill) and are not stored; K past C reads zeros on both
+// operands.  All waits are bounded: on expiry the CTA records
 // SVA_ERR_DEVICE_TIMEOUT, drains its own copies and MMAs, frees TMEM and
 // exits.
 #include <mutex>
@@ -83,6 +84,17 @@ __device__ __forceinline__ uint32_t rotate2_bf16(float x, float y, float2 cs) {
   const float rx = __fmaf_rn(x, cs.x, -(y * cs.y));
   const float ry = __fmaf_rn(x, cs.y, y * cs.x);
   return pack2_bf16(rx, ry);
+}
+
+// Tile store shared -> global through a 3D tensor map (bulk-group
+// completion); elements outside the tensor's extent are not written.
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* map, uint32_t src, int32_t c0,
+                                             int32_t c1, int32_t c2) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(src), "r"(c0), "r"(c1), "r"(c2)
+      : "memory");
 }
 
 __device__ __forceinline__ void proj_timeout(const ProjParams& p, volatile int* abort_flag) {
@@ -329,6 +341,18 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
         uint64_t rowp[4];  // the cache rows this lane writes in store_rows
 #pragma unroll
         for (int j = 0; j < 4; ++j) rowp[j] = __shfl_sync(0xffffffffu, cdst, j * 8 + (lane >> 2));
+        // K' and V: when this warp's 32 rows are tokens of one node (rows past
+        // that node's T, only possible for the last node, are clipped by the
+        // slot-pool map), a chunk leaves by one tile store at (column, token
+        // u0, (slot, K|V, head)); a chunk whose rows straddle two nodes goes
+        // row by row.
+        int u0 = 0, kv_plane = -1;  // first token; (slot * 2 + K|V) * H, or -1: row by row
+        if (tensor != 0 && y0 < p.rows) {
+          const int n0 = y0 / rp.T;
+          u0 = y0 - n0 * rp.T;
+          if (u0 + 32 <= rp.T || n0 == rp.n_nodes - 1)
+            kv_plane = (rp.nodes[n0].slot * 2 + (tensor == 2 ? 1 : 0)) * rp.H;
+        }
         // The 32-column chunk ci of every head in the item uses the same 16
         // (cos, sin) pairs, fetched once per chunk index (the next one while
         // the current one is rotated); this warp takes the chunk indices of
@@ -383,7 +407,17 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
               store_tile(stage(w, true), &p.tmap_out[0], c0 + c * 32, y0);  // Q' token-major
             } else {
               const int head = (c0 + c * 32) / rp.d;
-              store_rows(stage(w, false), rowp, (size_t)head * rp.Tpad * rp.d + (size_t)ci * 32);
+              if (kv_plane >= 0) {
+                const uint32_t buf = stage(w, true);
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                  tma_store_3d(&p.tmap_out[1], buf, ci * 32, u0, kv_plane + head);
+                  bulk_commit_group();
+                }
+              } else {
+                store_rows(stage(w, false), rowp, (size_t)head * rp.Tpad * rp.d + (size_t)ci * 32);
+              }
             }
           }
         }

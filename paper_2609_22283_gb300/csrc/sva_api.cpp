@@ -3,7 +3,7 @@
 // Owns the (seq, chunk, level) -> slot table of the KV cache (Section 3.2),
 // the integer rules of context selection (Eq. 2-3), pipeline rounds (Eq. 6)
 // and availability (Eq. 7), the validation of every launch, the TMA
-// descriptors, and the launches of the two kernels.  Device memory is always
+// descriptors, and the launches of the kernels.  Device memory is always
 // the caller's.
 #include <algorithm>
 #include <climits>
@@ -903,6 +903,21 @@ sva_status project(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const v
                       CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
       if (r != CUDA_SUCCESS)
         return fail(SVA_ERR_CUDA, "cuTensorMapEncodeTiled(output %d) failed: %d", i, (int)r);
+    }
+    if (rope) {
+      // K' and V into the slot pool: rows of one (slot, K|V, head) are the
+      // tokens [0, T) of that slot (the padding rows up to Tpad untouched)
+      const sva_geometry& g0 = c->g;
+      cuuint64_t dims[3] = {(cuuint64_t)g0.head_dim, (cuuint64_t)c->L.T,
+                            (cuuint64_t)g0.num_slots * 2 * g0.num_heads};
+      cuuint64_t strides[2] = {(cuuint64_t)g0.head_dim * 2, (cuuint64_t)c->L.Tpad * g0.head_dim * 2};
+      cuuint32_t box[3] = {32, 32, 1};
+      cuuint32_t es3[3] = {1, 1, 1};
+      CUresult r = fn(&p.tmap_out[1], CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, c->base, dims, strides,
+                      box, es3, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B,
+                      CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+      if (r != CUDA_SUCCESS)
+        return fail(SVA_ERR_CUDA, "cuTensorMapEncodeTiled(slot pool) failed: %d", (int)r);
     }
   }
   if (rope) {
