@@ -9,8 +9,8 @@ namespace sva {
 // The QKV projection y = x W^T + b split into q, k, v (sva_qkv_project).
 struct ProjParams {
   CUtensorMap tmap_x;   // x as 2D (C, rows), box (64, 128), 128B swizzle
-  CUtensorMap tmap_w;   // weight as 2D (C, 3N), box (64, BN), 128B swizzle
-  CUtensorMap tmap_wh;  // the same weight with box (64, BN / 2): half-width items
+  CUtensorMap tmap_w;   // weight as 2D (C, 3N), box (64, BN / 2): one CTA's half of a tile
+  CUtensorMap tmap_wh;  // the same weight with box (64, BN / 4): half-width items
   // out[i] as 2D (N, rows), box (32, 32), 64B swizzle: the epilogue's tile
   // stores.  With rope_on: tmap_out[0] is Q' token-major, tmap_out[1] the
   // slot pool as 3D (d, T, num_slots * 2 * H) with the (slot, K|V, head)
@@ -20,10 +20,11 @@ struct ProjParams {
   void* out[3];         // q, k, v: bf16 [rows][N]
   int* status;          // device status word
   int32_t rows, C, N;   // N = H * d outputs per tensor
-  int32_t n_mtiles, n_ntiles, n_kblocks;
-  // Work items: output tile t = m * n_ntiles + n for items 0..n_whole-1; the
-  // tiles n_whole.. as two half-width items each (columns [0, BN/2) and
-  // [BN/2, BN) of the tile), items n_whole.. n_items-1.
+  int32_t n_mtiles, n_ntiles, n_kblocks;  // 256-row tiles, BN-column tiles, 64-wide K blocks
+  // Work items: output tiles 0..n_whole-1 whole (tile t in the grouped raster
+  // of the kernel: groups of 16 row tiles, row tile fastest); the tiles
+  // n_whole.. as two half-width items each (columns [0, BN/2) and [BN/2, BN)
+  // of the tile), items n_whole.. n_items-1.
   int32_t n_items, n_whole;
   uint64_t timeout_ns;
   // Fused RoPE + cache scatter epilogue (sva_qkv_project_rope): q and k are
@@ -35,6 +36,12 @@ struct ProjParams {
   RopeParams rope;
 };
 
+// `grid` CTAs in clusters of two (grid even): each pair computes 256-row
+// tiles with two-SM MMAs.
 cudaError_t launch_qkv_project(const ProjParams& p, int block_n, int grid, cudaStream_t s);
+
+// Clusters of two CTAs of the projection kernel that can be resident at once
+// on the current device (one CTA per SM): the persistent grid's pair count.
+cudaError_t qkv_project_max_pairs(int block_n, int* pairs);
 
 }  // namespace sva

@@ -4,20 +4,34 @@
 // contraction, so it runs on the tensor cores:
 //
 //   bf16 x [rows][C] (A, K-major) times bf16 W [3N][C] (B, K-major) into an
-//   fp32 accumulator in TMEM, 128 x BN output tiles (BN = 256, or 128 when
-//   N = H*d is not a multiple of 256), 64-wide K blocks through a 4-stage
-//   TMA ring.
+//   fp32 accumulator in TMEM, 256 x BN output tiles (BN = 256, or 128 when
+//   N = H*d is not a multiple of 256), 64-wide K blocks through a TMA ring.
 //
-// Persistent CTAs (one per SM) walk a list of work items; two TMEM
+// Each tile is computed by a pair of CTAs (a cluster of two) with two-SM
+// MMAs (tcgen05 cta_group::2, M = 256): CTA r of the pair loads rows
+// [128 r, 128 r + 128) of the tile's x rows and rows [r BN/2, (r+1) BN/2) of
+// its W rows into the same shared-memory offsets, the even CTA issues the
+// MMAs, and each CTA's tensor memory receives its own 128 accumulator rows.
+// Per SM a K block then brings 16 KB of x and BN/2 x 64 of W from L2 (32 KB
+// at BN = 256) for 512 tensor cycles, against 48 KB for a one-SM 128 x 256
+// tile.  Both CTAs' copies count toward the even CTA's stage barrier; the
+// MMA commits free the stage in each CTA and hand the accumulator to each
+// CTA's epilogue; the odd CTA's epilogue warps arrive remotely on the even
+// CTA's accumulator-free barrier.
+//
+// Persistent pairs (one CTA per SM) walk a list of work items; two TMEM
 // accumulators let the epilogue of one item (TMEM -> + bias -> bf16 ->
-// global) overlap the main loop of the next.  Items are output tiles with
-// the column tile varying fastest, so the CTAs running at one time read the
-// same few x row tiles (shared through L2) and all of W (which stays in L2).
-// When the tiles do not fill the last round of CTAs, the tiles of that round
-// are split into two half-width items (BN / 2 columns), so that the last
-// round takes half as long.
+// global) overlap the main loop of the next.  Items are output tiles in
+// groups of up to 16 row tiles, the row tile varying fastest inside a group:
+// the pairs running at one time share each W column tile through L2, and a
+// group's x rows (at most 16 x 256 rows) stay in L2 while the group sweeps
+// the columns, so that W is read from HBM once per group even where it does
+// not fit in L2.  When the tiles do not fill the last round of pairs, the
+// tiles of that round are split into two half-width items (BN / 2 columns),
+// so that the last round takes half as long.
 //   warp 0      TMA producer (x and W tiles, 128-byte swizzle);
-//   warp 1      TMEM owner and MMA issuer (whole warp, one elected lane);
+//   warp 1      TMEM owner (both CTAs) and MMA issuer (even CTA; whole warp,
+//               one elected lane);
 //   warps 4-11  epilogue: two warps per TMEM lane quarter, one output row per
 //               thread, the two warps of a quarter taking alternate 32-column
 //               chunks.  Each chunk (32 rows x 64 bytes) is staged in the
@@ -51,27 +65,31 @@ namespace {
 using namespace ptx;
 
 constexpr int kProjThreads = 384;
-constexpr int kStages = 4;
-constexpr int kBM = 128;
+constexpr int kMaxStages = 8;
+constexpr int kBM = 128;       // accumulator rows per CTA (a pair's tile has 256)
 constexpr int kBK = 64;
 constexpr int kEpiWarps = 8;
+constexpr int kGroupM = 16;    // row tiles per raster group
 constexpr int kChunkBytes = 32 * 64;  // one staged 32 x 32 bf16 output chunk
 
 template <int BN>
 struct ProjCfg {
-  static constexpr int kABytes = kBM * kBK * 2;  // 16 KB
-  static constexpr int kBBytes = BN * kBK * 2;   // 32 KB at BN = 256
+  static constexpr int kABytes = kBM * kBK * 2;        // 16 KB of x rows per CTA
+  static constexpr int kBBytes = (BN / 2) * kBK * 2;   // this CTA's half of the W rows
   static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStages = BN == 256 ? 6 : 8;
   static constexpr int kOutBytes = kEpiWarps * 2 * kChunkBytes;  // output staging, 32 KB
   static constexpr int kSmemBytes = kStages * kStageBytes + kOutBytes + 1024;  // + alignment slack
   static constexpr uint32_t kTmemCols = 2 * BN;                   // two accumulators
+  static_assert(kStages <= kMaxStages, "stage barriers");
+  static_assert(kSmemBytes + 256 <= 227 * 1024, "shared memory per CTA");
 };
 
 struct ProjBars {
-  uint64_t full[kStages];
-  uint64_t empty[kStages];
-  uint64_t acc_full[2];
-  uint64_t acc_empty[2];  // one arrival per epilogue warp
+  uint64_t full[kMaxStages];   // even CTA: both CTAs' copies of a stage landed
+  uint64_t empty[kMaxStages];  // this CTA's stage was read by the MMAs
+  uint64_t acc_full[2];        // the accumulator of an item is complete
+  uint64_t acc_empty[2];       // even CTA: both CTAs' epilogues read it (16 arrivals)
   uint64_t drain;
 };
 
@@ -116,14 +134,22 @@ __device__ __forceinline__ Item item_of(const ProjParams& p, int i) {
     t = p.n_whole + ((i - p.n_whole) >> 1);
     it.half = (i - p.n_whole) & 1;
   }
-  it.m = t / p.n_ntiles;
-  it.n = t - it.m * p.n_ntiles;
+  // tile t of the raster: groups of kGroupM row tiles (the last may be
+  // smaller), the row tile varying fastest inside a group
+  const int per_group = kGroupM * p.n_ntiles;
+  const int g = t / per_group;
+  const int r = t - g * per_group;
+  const int gm = min(kGroupM, p.n_mtiles - g * kGroupM);
+  const int n = r / gm;
+  it.m = g * kGroupM + (r - n * gm);
+  it.n = n;
   return it;
 }
 
 template <int BN>
 __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __grid_constant__ ProjParams p) {
   using C = ProjCfg<BN>;
+  constexpr int kStages = C::kStages;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
@@ -133,6 +159,9 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();  // 0: issues the MMAs of the pair
+  const int pair = blockIdx.x >> 1;
+  const int n_pairs = gridDim.x >> 1;
 
   if (threadIdx.x == 0) {
     abort_flag = 0;
@@ -142,17 +171,18 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(&bars.acc_full[b], 1);
-      mbar_init(&bars.acc_empty[b], kEpiWarps);
+      mbar_init(&bars.acc_empty[b], 2 * kEpiWarps);
     }
     mbar_init(&bars.drain, 1);
     fence_mbar_init();
   }
   if (warp == 1) {
-    tmem_alloc(&tmem_base_sh, C::kTmemCols);
-    tmem_relinquish();
+    tmem_alloc_pair(&tmem_base_sh, C::kTmemCols);
+    tmem_relinquish_pair();
   }
   tc_fence_before();
-  __syncthreads();
+  // both CTAs' barriers are initialised before either signals the other's
+  cluster_sync();
   tc_fence_after();
   const uint32_t tbase = tmem_base_sh;
   const uint64_t tmo = p.timeout_ns;
@@ -164,11 +194,15 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
       prefetch_tmap(&p.tmap_x);
       prefetch_tmap(&p.tmap_w);
       prefetch_tmap(&p.tmap_wh);
-      for (int i = blockIdx.x; i < p.n_items; i += gridDim.x) {
+      const uint32_t full0 = mapa_shared(smem_u32(&bars.full[0]), 0);  // even CTA's barriers
+      for (int i = pair; i < p.n_items; i += n_pairs) {
         const Item it = item_of(p, i);
         const bool half = it.half >= 0;
+        // this CTA's part of the stage: its 128 x rows and its half of the W rows
         const uint32_t bytes = C::kABytes + (half ? C::kBBytes / 2 : C::kBBytes);
-        const int w_row = it.n * BN + (half ? it.half * (BN / 2) : 0);
+        const int x_row = it.m * 2 * kBM + (int)rank * kBM;
+        const int w_row = it.n * BN + (half ? it.half * (BN / 2) + (int)rank * (BN / 4)
+                                            : (int)rank * (BN / 2));
         bool ok = true;
         for (int kb = 0; kb < p.n_kblocks; ++kb, ++issued) {
           const int s = issued % kStages;
@@ -179,54 +213,65 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
             break;
           }
           uint8_t* sa = smem + s * C::kStageBytes;
-          mbar_arrive_expect_tx(&bars.full[s], bytes);
-          tma_load_2d(sa, &p.tmap_x, &bars.full[s], kb * kBK, it.m * kBM);
-          tma_load_2d(sa + C::kABytes, half ? &p.tmap_wh : &p.tmap_w, &bars.full[s], kb * kBK,
-                      w_row);
+          const uint32_t full = full0 + (uint32_t)(s * sizeof(uint64_t));
+          if (rank == 0) mbar_arrive_expect_tx(&bars.full[s], 2 * bytes);  // both CTAs' bytes
+          tma_load_2d_pair(sa, &p.tmap_x, full, kb * kBK, x_row);
+          tma_load_2d_pair(sa + C::kABytes, half ? &p.tmap_wh : &p.tmap_w, full, kb * kBK, w_row);
         }
         if (!ok) break;
       }
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    constexpr uint32_t idesc_whole = idesc_bf16_f32(kBM, BN, false);
-    constexpr uint32_t idesc_half = idesc_bf16_f32(kBM, BN / 2, false);
-    const uint64_t dA = sdesc_sw128(smem_u32(smem), 16, 1024);
-    const uint64_t dB = sdesc_sw128(smem_u32(smem + C::kABytes), 16, 1024);
-    constexpr uint64_t kStageStep = (uint64_t)(C::kStageBytes >> 4);
-    auto wait = [&](uint64_t* bar, uint32_t parity) {
-      return __all_sync(0xffffffffu, mbar_wait(bar, parity, &abort_flag, tmo));
-    };
-    bool ok = true;
-    int k_it = 0, tc = 0;
-    for (int i = blockIdx.x; ok && i < p.n_items; i += gridDim.x, ++tc) {
-      const uint32_t idesc = item_of(p, i).half >= 0 ? idesc_half : idesc_whole;
-      const int acc = tc & 1;
-      if (!wait(&bars.acc_empty[acc], ((uint32_t)(tc >> 1) & 1u) ^ 1u)) {
-        ok = false;
-        break;
-      }
-      tc_fence_after();
-      const uint32_t dcol = tbase + (uint32_t)(acc * BN);
-      for (int kb = 0; kb < p.n_kblocks; ++kb, ++k_it) {
-        const int s = k_it % kStages;
-        if (!wait(&bars.full[s], (uint32_t)(k_it / kStages) & 1u)) {
+    if (rank == 0) {
+      constexpr uint32_t idesc_whole = idesc_bf16_f32(2 * kBM, BN, false);
+      constexpr uint32_t idesc_half = idesc_bf16_f32(2 * kBM, BN / 2, false);
+      const uint64_t dA = sdesc_sw128(smem_u32(smem), 16, 1024);
+      const uint64_t dB = sdesc_sw128(smem_u32(smem + C::kABytes), 16, 1024);
+      constexpr uint64_t kStageStep = (uint64_t)(C::kStageBytes >> 4);
+      const uint32_t empty_own = smem_u32(&bars.empty[0]);
+      const uint32_t empty_peer = mapa_shared(empty_own, 1);
+      const uint32_t accf_own = smem_u32(&bars.acc_full[0]);
+      const uint32_t accf_peer = mapa_shared(accf_own, 1);
+      auto wait = [&](uint64_t* bar, uint32_t parity) {
+        return __all_sync(0xffffffffu, mbar_wait(bar, parity, &abort_flag, tmo));
+      };
+      bool ok = true;
+      int k_it = 0, tc = 0;
+      for (int i = pair; ok && i < p.n_items; i += n_pairs, ++tc) {
+        const uint32_t idesc = item_of(p, i).half >= 0 ? idesc_half : idesc_whole;
+        const int acc = tc & 1;
+        if (!wait(&bars.acc_empty[acc], ((uint32_t)(tc >> 1) & 1u) ^ 1u)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint64_t a = dA + (uint64_t)s * kStageStep;
-        const uint64_t b = dB + (uint64_t)s * kStageStep;
+        const uint32_t dcol = tbase + (uint32_t)(acc * BN);
+        for (int kb = 0; kb < p.n_kblocks; ++kb, ++k_it) {
+          const int s = k_it % kStages;
+          if (!wait(&bars.full[s], (uint32_t)(k_it / kStages) & 1u)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint64_t a = dA + (uint64_t)s * kStageStep;
+          const uint64_t b = dB + (uint64_t)s * kStageStep;
 #pragma unroll
-        for (int kk = 0; kk < kBK / 16; ++kk)  // 32 bytes of K per MMA inside the swizzle atom
-          mma_ss_warp(dcol, a + (uint64_t)(kk * 2), b + (uint64_t)(kk * 2), idesc,
-                      (kb > 0 || kk > 0) ? 1u : 0u);
-        mma_commit_warp(&bars.empty[s]);  // the stage is free once these MMAs have read it
+          for (int kk = 0; kk < kBK / 16; ++kk)  // 32 bytes of K per MMA inside the swizzle atom
+            mma_ss_pair_warp(dcol, a + (uint64_t)(kk * 2), b + (uint64_t)(kk * 2), idesc,
+                             (kb > 0 || kk > 0) ? 1u : 0u);
+          // the stage is free in each CTA once these MMAs have read it
+          const uint32_t off = (uint32_t)(s * sizeof(uint64_t));
+          mma_commit_pair_warp(empty_own + off);
+          mma_commit_pair_warp(empty_peer + off);
+        }
+        if (!ok) break;
+        const uint32_t off = (uint32_t)(acc * sizeof(uint64_t));
+        mma_commit_pair_warp(accf_own + off);
+        mma_commit_pair_warp(accf_peer + off);
       }
-      if (!ok) break;
-      mma_commit_warp(&bars.acc_full[acc]);
+      if (!ok && lane == 0) proj_timeout(p, &abort_flag);
     }
-    if (!ok && lane == 0) proj_timeout(p, &abort_flag);
   } else if (warp >= 4) {
     // ------------------------------------------------------------ epilogue
     const int q4 = warp & 3;           // TMEM lane quarter this warp may access
@@ -288,7 +333,8 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
     };
     bool ok = true;
     int tc = 0;
-    for (int i = blockIdx.x; ok && i < p.n_items; i += gridDim.x, ++tc) {
+    const uint32_t acce0 = mapa_shared(smem_u32(&bars.acc_empty[0]), 0);  // even CTA's
+    for (int i = pair; ok && i < p.n_items; i += n_pairs, ++tc) {
       const Item it = item_of(p, i);
       const int width = it.half >= 0 ? BN / 2 : BN;  // output columns of this item
       const int acc = tc & 1;
@@ -303,7 +349,7 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
       const int col = it.n * BN + (it.half > 0 ? BN / 2 : 0);  // output column in [0, 3N)
       const int tensor = col / p.N;      // q, k or v
       const int c0 = col - tensor * p.N;  // column inside that tensor
-      const int y0 = it.m * kBM + q4 * 32;  // first output row of this warp
+      const int y0 = it.m * 2 * kBM + (int)rank * kBM + q4 * 32;  // first output row of this warp
       // 32 accumulator columns of this row: TMEM -> registers, plus the bias
       auto load_chunk = [&](int c, uint32_t (&r)[32], float (&bv)[32]) {
         tmem_ld32(tbase + lane_off + (uint32_t)(acc * BN + c * 32), r);
@@ -323,7 +369,7 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
       if (p.rope_on) {
         // Fused RoPE: this row's node, token and position, and where K' / V go
         const RopeParams& rp = p.rope;
-        const long long grow = (long long)it.m * kBM + row;
+        const long long grow = (long long)it.m * 2 * kBM + (int)rank * kBM + row;
         int tpos = 0, hh = 0, ww = 0;
         uint64_t cdst = 0;  // (slot, K or V, head 0, token u, dim 0) of the cache; 0 past `rows`
         if (grow < p.rows) {
@@ -437,10 +483,11 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
         }
       }
       // The MMA warp may overwrite this accumulator once every epilogue warp
-      // has read its part (each thread waited for its own TMEM loads).
+      // of both CTAs has read its part (each thread waited for its own TMEM
+      // loads).
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&bars.acc_empty[acc]);
+      if (lane == 0) mbar_arrive_cluster(acce0 + (uint32_t)(acc * sizeof(uint64_t)));
     }
     // the bulk stores read this CTA's shared memory and must be complete
     // before it exits
@@ -450,25 +497,35 @@ __global__ void __launch_bounds__(kProjThreads, 1) qkv_project_kernel(const __gr
   }
 
   // ---------------------------------------------------------------- teardown
-  __syncwarp();
-  tc_fence_before();
-  __syncthreads();
-  if (abort_flag) {
-    // Some wait expired: wait (bounded, ignoring the abort flag) for the
-    // copies this CTA started and for every MMA it issued before exiting.
+  // Every MMA that reads this CTA's stages has completed, and its commits
+  // have arrived here, once the last round of this CTA's stages is free
+  // again (bounded wait).  After a timeout the even CTA also waits for its
+  // stage barriers, whose phases count both CTAs' copies, and for every MMA
+  // it issued.
+  if (warp == 0 && lane == 0) {
     const int zero = 0;
-    if (warp == 0 && lane == 0) {
-      for (int i = (issued > kStages ? issued - kStages : 0); i < issued; ++i)
+    for (int i = (issued > kStages ? issued - kStages : 0); i < issued; ++i) {
+      mbar_wait(&bars.empty[i % kStages], (uint32_t)(i / kStages) & 1u, &zero, tmo);
+      if (abort_flag && rank == 0)
         mbar_wait(&bars.full[i % kStages], (uint32_t)(i / kStages) & 1u, &zero, tmo);
-    } else if (warp == 1) {
-      mma_commit_warp(&bars.drain);
-      mbar_wait(&bars.drain, 0, &zero, tmo);
     }
   }
   __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (abort_flag && rank == 0 && warp == 1) {
+    const int zero = 0;
+    mma_commit_pair_warp(smem_u32(&bars.drain));
+    mbar_wait(&bars.drain, 0, &zero, tmo);
+  }
+  __syncwarp();
+  tc_fence_before();
+  // neither CTA leaves (or frees tensor memory) while the other may still
+  // signal its barriers or have MMAs read its shared memory
+  cluster_sync();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tbase, C::kTmemCols);
+    tmem_dealloc_pair(tbase, C::kTmemCols);
   }
 }
 
@@ -491,22 +548,73 @@ cudaError_t configure_bn(int dev) {
 }
 
 template <int BN>
+void pair_launch_config(cudaLaunchConfig_t* cfg, cudaLaunchAttribute* attr, int grid,
+                        cudaStream_t s) {
+  *cfg = cudaLaunchConfig_t{};
+  cfg->gridDim = dim3((unsigned)grid, 1, 1);
+  cfg->blockDim = dim3(kProjThreads, 1, 1);
+  cfg->dynamicSmemBytes = ProjCfg<BN>::kSmemBytes;
+  cfg->stream = s;
+  attr->id = cudaLaunchAttributeClusterDimension;
+  attr->val.clusterDim.x = 2;
+  attr->val.clusterDim.y = 1;
+  attr->val.clusterDim.z = 1;
+  cfg->attrs = attr;
+  cfg->numAttrs = 1;
+}
+
+template <int BN>
 cudaError_t launch_bn(const ProjParams& p, int grid, cudaStream_t s) {
-  using C = ProjCfg<BN>;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   e = configure_bn<BN>(dev);
   if (e != cudaSuccess) return e;
-  qkv_project_kernel<BN><<<grid, kProjThreads, C::kSmemBytes, s>>>(p);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg;
+  cudaLaunchAttribute attr;
+  pair_launch_config<BN>(&cfg, &attr, grid, s);
+  return cudaLaunchKernelEx(&cfg, qkv_project_kernel<BN>, p);
+}
+
+// Clusters of two (one CTA per SM) that can be resident at once on the
+// current device, looked up once per device and instance.
+template <int BN>
+cudaError_t max_pairs_bn(int* out) {
+  static std::mutex mu;
+  static int pairs[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  e = configure_bn<BN>(dev);
+  if (e != cudaSuccess) return e;
+  std::lock_guard<std::mutex> lock(mu);
+  if (pairs[dev] == 0) {
+    cudaLaunchConfig_t cfg;
+    cudaLaunchAttribute attr;
+    pair_launch_config<BN>(&cfg, &attr, 2, nullptr);
+    int n = 0;
+    e = cudaOccupancyMaxActiveClusters(&n, qkv_project_kernel<BN>, &cfg);
+    if (e != cudaSuccess) return e;
+    if (n < 1) return cudaErrorInvalidConfiguration;
+    pairs[dev] = n;
+  }
+  *out = pairs[dev];
+  return cudaSuccess;
 }
 
 }  // namespace
 
 cudaError_t launch_qkv_project(const ProjParams& p, int block_n, int grid, cudaStream_t s) {
+  if (grid < 2 || grid % 2 != 0) return cudaErrorInvalidValue;
   if (block_n == 256) return launch_bn<256>(p, grid, s);
   if (block_n == 128) return launch_bn<128>(p, grid, s);
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t qkv_project_max_pairs(int block_n, int* pairs) {
+  if (block_n == 256) return max_pairs_bn<256>(pairs);
+  if (block_n == 128) return max_pairs_bn<128>(pairs);
   return cudaErrorInvalidValue;
 }
 

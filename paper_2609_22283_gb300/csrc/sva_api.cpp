@@ -879,10 +879,11 @@ sva_status project(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const v
     if (r != CUDA_SUCCESS) return fail(SVA_ERR_CUDA, "cuTensorMapEncodeTiled(x) failed: %d", (int)r);
   }
   for (int half = 0; half < 2; ++half) {
-    // W tiles of a whole item (BN rows) and of a half-width item (BN / 2)
+    // one CTA's half of the W rows of a whole item (BN / 2 rows) and of a
+    // half-width item (BN / 4)
     cuuint64_t dims[2] = {(cuuint64_t)in_features, (cuuint64_t)3 * N};
     cuuint64_t strides[1] = {(cuuint64_t)in_features * 2};
-    cuuint32_t box[2] = {64, (cuuint32_t)(half ? bn / 2 : bn)};
+    cuuint32_t box[2] = {64, (cuuint32_t)(half ? bn / 4 : bn / 2)};
     CUresult r = fn(half ? &p.tmap_wh : &p.tmap_w, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
                     const_cast<void*>(weight), dims, strides, box, es,
                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -962,23 +963,26 @@ sva_status project(sva_cache* c, const sva_node* nodes, int32_t n_nodes, const v
   p.rows = rows;
   p.C = in_features;
   p.N = N;
-  p.n_mtiles = (rows + 127) / 128;
+  p.n_mtiles = (rows + 255) / 256;
   p.n_ntiles = 3 * N / bn;
   p.n_kblocks = (in_features + 63) / 64;
   p.timeout_ns = c->timeout_ns;
-  // One CTA per SM walks the items.  The tiles of a partial last round are
-  // split into two half-width items when the halves fit one round (and, for
-  // the fused RoPE epilogue, still cover whole heads), so that the last round
-  // takes half as long.
-  const long long sms = c->num_sms;
+  // One pair of CTAs per two SMs walks the items.  The tiles of a partial
+  // last round are split into two half-width items when the halves fit one
+  // round (and, for the fused RoPE epilogue, still cover whole heads), so
+  // that the last round takes half as long.
+  int max_pairs = 0;
+  cudaError_t e = sva::qkv_project_max_pairs(bn, &max_pairs);
+  if (e != cudaSuccess) return cuda_fail(e, "qkv_project occupancy");
+  const long long pairs = std::max(1, std::min(max_pairs, c->num_sms / 2));
   const long long tiles = (long long)p.n_mtiles * p.n_ntiles;
   if (tiles > INT32_MAX / 2) return fail(SVA_ERR_CAPACITY, "%lld output tiles", tiles);
-  const long long rest = tiles % sms;
-  const bool split_tail = rest > 0 && 2 * rest <= sms && (!rope || (bn / 2) % g.head_dim == 0);
+  const long long rest = tiles % pairs;
+  const bool split_tail = rest > 0 && 2 * rest <= pairs && (!rope || (bn / 2) % g.head_dim == 0);
   p.n_whole = (int32_t)(split_tail ? tiles - rest : tiles);
   p.n_items = (int32_t)(split_tail ? tiles + rest : tiles);
-  const int grid = (int)std::min<long long>(p.n_items, sms);
-  cudaError_t e = sva::launch_qkv_project(p, bn, grid, reinterpret_cast<cudaStream_t>(s));
+  const int grid = 2 * (int)std::min<long long>(p.n_items, pairs);
+  e = sva::launch_qkv_project(p, bn, grid, reinterpret_cast<cudaStream_t>(s));
   if (e != cudaSuccess) return cuda_fail(e, "qkv_project launch");
   if (rope)
     for (int i = 0; i < n_nodes; ++i) c->slots[nodes[i].own_slot].resident = true;
