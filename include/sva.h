@@ -218,8 +218,9 @@ sva_status sva_rope_kv_write_qknorm(sva_cache* c, const sva_node* nodes, int32_t
  * in_features a positive multiple of 8; H*d a multiple of 128; every pointer
  * 16-byte aligned and in device memory of the cache's device (a host or
  * another GPU's pointer is rejected with INVALID_ARGUMENT before anything is
- * launched).  Each CTA loads its own operand tiles from this GPU's memory
- * (no copy is shared between CTAs).  Stream-ordered; a device timeout is
+ * launched).  Runs on pairs of CTAs (clusters of two) with two-SM MMAs;
+ * each CTA loads its own operand tiles from this GPU's memory (no copy
+ * writes more than one CTA).  Stream-ordered; a device timeout is
  * reported by sva_poll_device_status.  Errors: INVALID_ARGUMENT,
  * UNSUPPORTED (H*d), CUDA. */
 sva_status sva_qkv_project(sva_cache* c, const void* x, int32_t rows, int32_t in_features,

@@ -40,12 +40,14 @@ def _project(w, C, rows_sample=None, bias=True):
     outs = [torch.empty((w.n_nodes, w.T, w.H, w.d), dtype=torch.bfloat16, device=dev) for _ in range(3)]
     cache.qkv_project(xd, wd, bd, *outs)
     assert cache.poll() == 0
-    got = [o.float().cpu().numpy().reshape(-1, w.H, w.d) for o in outs]
-    xs = x.double().numpy().reshape(-1, C)
-    idx = np.arange(xs.shape[0]) if rows_sample is None else np.asarray(rows_sample)
-    ref = oracle.qkv_project(xs[idx], wt.double().numpy(), b.double().numpy() if bias else None, heads=w.H)
+    n_rows = w.n_nodes * w.T
+    idx = np.arange(n_rows) if rows_sample is None else np.asarray(rows_sample)
+    sel = torch.from_numpy(idx).to(dev)
+    got = [o.view(n_rows, w.H, w.d).index_select(0, sel).float().cpu().numpy() for o in outs]
+    xs = x.reshape(n_rows, C)[torch.from_numpy(idx)].double().numpy()
+    ref = oracle.qkv_project(xs, wt.double().numpy(), b.double().numpy() if bias else None, heads=w.H)
     for t in range(3):
-        _check(got[t][idx], ref[t], f"{w.name} C={C} tensor {'qkv'[t]}")
+        _check(got[t], ref[t], f"{w.name} C={C} tensor {'qkv'[t]}")
     cache.close()
 
 
@@ -64,6 +66,26 @@ def test_wan_geometry_projection_sampled(oracle_mod):
     rng = np.random.default_rng(21)
     rows = sorted(set(rng.choice(w.n_nodes * w.T, 300, replace=False).tolist()) | {0, 18719, 18688, 127, 128})
     _project(w, 1536, rows)
+
+
+def test_clean1_rows_projection_split_tail_sampled(oracle_mod):
+    # 4680 rows: 19 tiles of 256 rows, the last with 72 (the odd CTA of the
+    # pair holds none of them); 342 tiles over the pairs leave a partial last
+    # round, split into half-width items
+    w = I.WORKLOADS["clean1"]
+    rng = np.random.default_rng(23)
+    edges = {0, 127, 128, 255, 256, 4351, 4352, 4607, 4608, 4679}
+    rows = sorted(set(rng.choice(w.n_nodes * w.T, 300, replace=False).tolist()) | edges)
+    _project(w, 1536, rows)
+
+
+def test_14b_geometry_projection_sampled(oracle_mod):
+    # 8 x 4680 rows, 5120 -> 3 x 40 x 128: 147 row tiles in groups of 16 (a
+    # weight larger than the L2), 80 K blocks
+    w = I.WORKLOADS["stress14b"]
+    rng = np.random.default_rng(25)
+    rows = sorted(set(rng.choice(w.n_nodes * w.T, 48, replace=False).tolist()) | {0, 4095, 4096, 37439})
+    _project(w, 5120, rows)
 
 
 def test_projection_feeds_rope_and_attention(oracle_mod):
@@ -230,6 +252,30 @@ def test_fused_projection_rope_wan_geometry_sampled(oracle_mod):
     step, inp, q, x, wt, b, nodes = _fused(w, 1536)
     rng = np.random.default_rng(22)
     rows = [sorted(set(rng.choice(w.T, 60, replace=False).tolist()) | {0, 127, 128, 1559, 1560, w.T - 1})
+            for _ in range(w.n_nodes)]
+    _check_fused(w, step, q, _fused_reference(w, x, wt, b, rows), rows, nodes)
+    step.close()
+
+
+def test_fused_projection_rope_clean1_split_tail_sampled(oracle_mod):
+    # one node of 4680 rows: the partial last round of 256-row tiles is split
+    # into half-width items of one head each; the last tile holds 72 rows
+    w = I.WORKLOADS["clean1"]
+    step, inp, q, x, wt, b, nodes = _fused(w, 1536)
+    rng = np.random.default_rng(24)
+    rows = [sorted(set(rng.choice(w.T, 120, replace=False).tolist()) |
+                   {0, 255, 256, 4607, 4608, w.T - 1})]
+    _check_fused(w, step, q, _fused_reference(w, x, wt, b, rows), rows, nodes)
+    step.close()
+
+
+def test_fused_projection_rope_14b_geometry_sampled(oracle_mod):
+    # 8 nodes x 4680 rows, 5120 -> 3 x 40 x 128; chunks of 32 rows that
+    # straddle two nodes go row by row
+    w = I.WORKLOADS["stress14b"]
+    step, inp, q, x, wt, b, nodes = _fused(w, 5120)
+    rng = np.random.default_rng(26)
+    rows = [sorted(set(rng.choice(w.T, 16, replace=False).tolist()) | {0, 4671, w.T - 1})
             for _ in range(w.n_nodes)]
     _check_fused(w, step, q, _fused_reference(w, x, wt, b, rows), rows, nodes)
     step.close()
