@@ -648,10 +648,28 @@ def time_projection(step, w, dev, flush, stream, peak, world, fused=False):
     ms = reduce_max(sum(a.elapsed_time(c) for a, c in ev) / K, world)
     flops = 2.0 * w.n_nodes * w.T * C * 3 * C
     tf = flops / (ms * 1e-3) / 1e12
-    return {"kernel": "qkv_project_kernel" + (" (fused RoPE + cache write)" if fused else ""),
-            "rows": w.n_nodes * w.T, "in_features": C,
-            "out_features": 3 * C, "ms": ms, "achieved": tf, "unit": "TFLOP/s",
-            "peak": peak, "frac": tf / peak, "launches": K}
+    res = {"kernel": "qkv_project_kernel" + (" (fused RoPE + cache write)" if fused else ""),
+           "rows": w.n_nodes * w.T, "in_features": C,
+           "out_features": 3 * C, "ms": ms, "achieved": tf, "unit": "TFLOP/s",
+           "peak": peak, "frac": tf / peak, "launches": K}
+    if not fused:
+        # context only: the library's bf16 matmul (cuBLAS) of the same shape,
+        # without the bias and the split into q, k, v, timed the same way
+        x2 = x.reshape(-1, C)
+        y = torch.empty((x2.shape[0], 3 * C), dtype=torch.bfloat16, device=dev)
+        for _ in range(3):
+            torch.matmul(x2, wt.t(), out=y)
+        torch.cuda.synchronize()
+        for e0, e1 in ev:
+            flush()
+            e0.record(stream)
+            torch.matmul(x2, wt.t(), out=y)
+            e1.record(stream)
+        torch.cuda.synchronize()
+        ms_ref = sum(a.elapsed_time(c) for a, c in ev) / K
+        res["cublas_same_shape"] = {"ms": ms_ref, "achieved": flops / (ms_ref * 1e-3) / 1e12,
+                                    "unit": "TFLOP/s", "note": "torch.matmul bf16, no bias; context"}
+    return res
 
 
 def compare_schedules(args):
