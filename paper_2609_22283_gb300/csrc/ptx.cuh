@@ -309,99 +309,6 @@ __device__ __forceinline__ void mma_commit_warp(uint64_t* bar) {
       : "memory");
 }
 
-// ---------------------------------------------------------------- CTA pairs
-//
-// Two-SM MMAs (cta_group::2): a cluster of two CTAs on neighbouring SMs; the
-// even-ranked CTA issues the MMAs, each reading its A rows and its half of
-// B from the shared memory of its own CTA (the same offsets in both), and
-// each CTA's tensor memory receives its own 128 accumulator rows.  Signals
-// between the two CTAs go to barriers named by their shared::cluster
-// address (mapa), one barrier per signal.
-
-__device__ __forceinline__ uint32_t cluster_ctarank() {
-  uint32_t r;
-  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-  return r;
-}
-
-// The shared::cluster address of the variable at `addr` (a shared::cta
-// address of this CTA) in the CTA of rank `rank` of the cluster.
-__device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
-  uint32_t r;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
-  return r;
-}
-
-__device__ __forceinline__ void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n"
-               "barrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-
-// Arrives once on a barrier of either CTA of the cluster (release at
-// cluster scope: this thread's earlier writes are visible to the waiter).
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
-               : "memory");
-}
-
-// tma_load_2d whose completion is counted on a barrier that may belong to
-// the peer CTA of the pair (`bar` is a shared::cluster address); the data
-// lands in this CTA's shared memory.
-__device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* map, uint32_t bar,
-                                                 int32_t c0, int32_t c1) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_u32(dst)),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1)
-      : "memory");
-}
-
-// Tensor-memory allocation for a CTA pair: one warp of each of the two CTAs
-// executes it; both get the same column base.
-__device__ __forceinline__ void tmem_alloc_pair(uint32_t* dst, uint32_t ncols) {
-  asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                   smem_u32(dst)),
-               "r"(ncols)
-               : "memory");
-}
-
-__device__ __forceinline__ void tmem_relinquish_pair() {
-  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
-}
-
-__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols) {
-  asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
-               : "memory");
-}
-
-// D[tmem of both CTAs] (+)= A[smem of both] * B[smem of both], M = 256 rows
-// (128 per CTA); issued by the even CTA only, warp-wide with one elected lane.
-__device__ __forceinline__ void mma_ss_pair_warp(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
-                                                 uint32_t idesc, uint32_t accumulate) {
-  asm volatile(
-      "{\n"
-      " .reg .pred p, e;\n"
-      " setp.ne.b32 p, %4, 0;\n"
-      " elect.sync _|e, 0xffffffff;\n"
-      " @e tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n"
-      "}\n" ::"r"(d_tmem),
-      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate)
-      : "memory");
-}
-
-// Arrives once on the barrier at shared::cluster address `bar` (this CTA's
-// or the peer's) when every tcgen05 operation this thread issued so far has
-// completed; warp-wide, one elected lane.
-__device__ __forceinline__ void mma_commit_pair_warp(uint32_t bar) {
-  asm volatile(
-      "{\n"
-      " .reg .pred e;\n"
-      " elect.sync _|e, 0xffffffff;\n"
-      " @e tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];\n"
-      "}\n" ::"r"(bar)
-      : "memory");
-}
-
 #define SVA_R8(i) "=r"(r[i]), "=r"(r[i + 1]), "=r"(r[i + 2]), "=r"(r[i + 3]), \
                   "=r"(r[i + 4]), "=r"(r[i + 5]), "=r"(r[i + 6]), "=r"(r[i + 7])
 #define SVA_W8(i) "r"(r[i]), "r"(r[i + 1]), "r"(r[i + 2]), "r"(r[i + 3]), \
