@@ -88,6 +88,26 @@ def test_14b_geometry_projection_sampled(oracle_mod):
     _project(w, 5120, rows)
 
 
+# 2 nodes of T = 100 tokens (one latent frame of 10 x 10), 2 heads of 128: 200
+# rows, so the one 256-row tile of a CTA pair gives the even CTA 128 rows and
+# the odd one 72 (the rows past 200 read zeros and are not stored); 256-wide
+# output tiles, 3 of them, whose last round is split into half-width items.
+ODD_HALF = I.Workload(name="oddhalf", seed=27, F=1, Hp=10, Wp=10, H=2, d=128, K=2, W=2,
+                      policy="prog", nodes=((0, 3, 2), (0, 2, 1)), prefilled=((0, 1, 0),))
+
+
+def test_projection_odd_cta_partly_filled(oracle_mod):
+    _project(ODD_HALF, 384)
+
+
+def test_fused_projection_rope_odd_cta_partly_filled(oracle_mod):
+    w = ODD_HALF
+    step, inp, q, x, wt, b, nodes = _fused(w, 384)
+    rows = [range(w.T)] * w.n_nodes
+    _check_fused(w, step, q, _fused_reference(w, x, wt, b, rows), rows, nodes)
+    step.close()
+
+
 def test_projection_feeds_rope_and_attention(oracle_mod):
     """x -> sva_qkv_project -> sva_rope_kv_write -> sva_attend_nodes against the
     oracle's projection (rounded to bf16 as stored) -> node_forward."""
