@@ -96,6 +96,15 @@ ODD_HALF = I.Workload(name="oddhalf", seed=27, F=1, Hp=10, Wp=10, H=2, d=128, K=
                       policy="prog", nodes=((0, 3, 2), (0, 2, 1)), prefilled=((0, 1, 0),))
 
 
+@pytest.mark.parametrize("wp", [1, 257])
+def test_projection_row_count_edges(oracle_mod, wp):
+    # one node of T = 1 or 257 tokens: a single row (the pair's odd CTA and
+    # 127 rows of the even one empty), and a second 256-row tile holding one row
+    w = I.Workload(name=f"rows{wp}", seed=28, F=1, Hp=1, Wp=wp, H=2, d=128, K=2, W=2,
+                   policy="clean", nodes=((0, 2, 1),), prefilled=((0, 1, 0),))
+    _project(w, 256)
+
+
 def test_projection_odd_cta_partly_filled(oracle_mod):
     _project(ODD_HALF, 384)
 
