@@ -117,6 +117,36 @@ def test_fused_projection_rope_odd_cta_partly_filled(oracle_mod):
     step.close()
 
 
+@pytest.mark.parametrize("name", ["clean1", "prog4"])
+def test_projection_bitwise_repeatable(name):
+    """The CTA pairs' signalling (both CTAs' copies counted on the even CTA's
+    stage barrier, commits to each CTA's barriers, remote accumulator-free
+    arrivals) leaves no race: repeated launches give the same bits, plain
+    and fused."""
+    w = I.WORKLOADS[name]
+    C = w.H * w.d
+    dev = torch.device("cuda")
+    x, wt, b = (t.to(dev).contiguous() for t in I.projection_inputs(w, C))
+    step = Step(w)
+    step.prefill(I.generate(w))
+    nodes, _ = step.node_table()
+    shape = (w.n_nodes, w.T, w.H, w.d)
+    runs = []
+    for _ in range(3):
+        outs = [torch.empty(shape, dtype=torch.bfloat16, device=dev) for _ in range(3)]
+        step.cache.qkv_project(x, wt, b, *outs)
+        q = torch.empty(shape, dtype=torch.bfloat16, device=dev)
+        step.cache.qkv_project_rope(nodes, x, wt, b, q)
+        own = [n.own_slot for n in nodes]
+        runs.append([o.view(torch.int16) for o in outs] +
+                    [q.view(torch.int16), step.cache.slot_pool()[own].view(torch.int16).clone()])
+    assert step.cache.poll() == 0
+    for r in runs[1:]:
+        for a, b0 in zip(r, runs[0]):
+            assert torch.equal(a, b0)
+    step.close()
+
+
 def test_projection_feeds_rope_and_attention(oracle_mod):
     """x -> sva_qkv_project -> sva_rope_kv_write -> sva_attend_nodes against the
     oracle's projection (rounded to bf16 as stored) -> node_forward."""
