@@ -137,6 +137,24 @@ def test_full_geometry_sampled(oracle_mod, name):
     print(f"\n{name} ({n_rows} rows): {stats}")
 
 
+@pytest.mark.parametrize("name", ["prog4", "stress14b"])
+def test_attention_bitwise_repeatable(name):
+    """Repeated launches on the same inputs give the same bits (no race in
+    the kernel's barriers, stage hand-back or lazy rescale)."""
+    w = I.WORKLOADS[name]
+    inp = I.generate(w)
+    step, q, out, lse = P.gpu_step(w, inp)
+    nodes, _ = step.node_table()
+    for _ in range(3):
+        again = torch.empty_like(out)
+        again_lse = torch.empty_like(lse)
+        step.cache.attend_nodes(nodes, q, again, again_lse, step.scale, check=False)
+        assert step.cache.poll() == 0
+        assert torch.equal(again.view(torch.int16), out.view(torch.int16))
+        assert torch.equal(again_lse.view(torch.int32), lse.view(torch.int32))
+    step.close()
+
+
 def test_clean5_serial_launches(oracle_mod):
     """The fully serial schedule of a chunk (Eq. 5) as the schedule comparison
     times it: each of the five nodes of chunk 20 (four updates, then the clean
